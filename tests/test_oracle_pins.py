@@ -1,0 +1,375 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself:
+values the paper prints, closed forms, invariants, textbook / library special cases
+and brute force on tiny inputs.  CPU only."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle as O
+import synth
+
+GOLD = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "paper_numbers.json")))
+
+
+def rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+# --------------------------------------------------------------------------- gates (Sec. 4.1)
+
+def test_block_and_ffn_gate_rule():
+    m = np.array([[0.3, -0.1, 0.0, 1e-30], [-2.0, 5.0, -0.0, 0.5]])
+    assert O.gates_from_soft_masks("block", m).tolist() == [[1, 0, 0, 1], [0, 1, 0, 1]]
+    assert O.gates_from_soft_masks("ffn", m).tolist() == [[1, 0, 0, 1], [0, 1, 0, 1]]
+
+
+def test_head_gate_rule_mean_of_head_entries():
+    # 3 heads of D_head = 4: mean positive / exactly zero / negative despite a large entry
+    m = np.array([0.1, 0.2, -0.05, 0.0,
+                  1.0, -1.0, 2.0, -2.0,
+                  5.0, -3.0, -3.0, -0.5])
+    assert O.gates_from_soft_masks("head", m, unit_size=4).tolist() == [1, 0, 0]
+
+
+def test_ffn_chunk_gate_expands_to_c_channels():
+    C = GOLD["ffn_chunk"]["value"]
+    g = O.ffn_channel_gate([1, 0, 1], C)
+    assert g.shape == (3 * C,)
+    assert g.tolist() == [1] * C + [0] * C + [1] * C
+
+
+def test_index_lists_follow_gates():
+    cfg = synth.tiny()
+    masks = synth.make_masks(cfg)
+    for s in range(4):
+        idx = O.compact_indices(cfg, masks, s, 0)
+        assert len(idx["heads"]) == cfg.heads_kept[s][0]
+        assert len(idx["chunks"]) == cfg.chunks_kept[s][0]
+        assert np.all(np.diff(idx["heads"]) > 0) and np.all(np.diff(idx["chunks"]) > 0)
+        # channels are whole heads / whole chunks of the retained units
+        assert set(idx["qk_rows"] // cfg.head_dim) == set(idx["heads"].tolist())
+        assert set(idx["ffn_ch"] // cfg.ffn_chunk) == set(idx["chunks"].tolist())
+        assert len(idx["ffn_ch"]) == 8 * len(idx["chunks"])
+
+
+def test_compact_panels_are_row_and_column_selections():
+    cfg = synth.tiny()
+    lw = synth.make_layer(cfg, 0)
+    masks = synth.make_masks(cfg)
+    idx = O.compact_indices(cfg, masks, 2, 0)
+    P = O.compact_panels(lw, idx)
+    hd = len(idx["heads"]) * cfg.head_dim
+    for i, h in enumerate(idx["heads"]):
+        for j in (0, cfg.head_dim - 1):
+            r = h * cfg.head_dim + j
+            np.testing.assert_array_equal(P["wqkv"][i * cfg.head_dim + j], lw["wq"][r])
+            np.testing.assert_array_equal(P["wqkv"][hd + i * cfg.head_dim + j], lw["wk"][r])
+            np.testing.assert_array_equal(P["wqkv"][2 * hd + i * cfg.head_dim + j], lw["wv"][r])
+            np.testing.assert_array_equal(P["wo"][:, i * cfg.head_dim + j], lw["wo"][:, r])
+    c0 = idx["chunks"][1]
+    np.testing.assert_array_equal(P["w_up"][8:16], lw["w_up"][c0 * 8:(c0 + 1) * 8])
+    np.testing.assert_array_equal(P["w_down"][:, 8:16], lw["w_down"][:, c0 * 8:(c0 + 1) * 8])
+
+
+# --------------------------------------------------------------------------- elementary ops
+
+def test_linear_orientation_out_in():
+    w = np.zeros((3, 5))
+    w[2, 4] = 1.0
+    x = rng().standard_normal((7, 5))
+    y = O.linear(x, w, np.array([0.0, 0.0, 0.5]))
+    np.testing.assert_allclose(y[:, 2], x[:, 4] + 0.5)
+    np.testing.assert_allclose(y[:, :2], 0.0)
+
+
+def test_modulation_affine_in_t_emb():
+    d = 8
+    r = rng(1)
+    w_t, b_t, e = r.standard_normal((6 * d, d)), r.standard_normal(6 * d), r.standard_normal((6, d))
+    np.testing.assert_allclose(O.modulation(w_t, b_t, e, np.zeros(d)), b_t.reshape(6, d) + e)
+    t = np.zeros(d)
+    t[3] = 1.0
+    np.testing.assert_allclose(O.modulation(w_t, b_t, e, t), (w_t[:, 3] + b_t).reshape(6, d) + e)
+
+
+def test_layer_norm_against_library_and_constant_row():
+    torch = pytest.importorskip("torch")
+    x = rng(2).standard_normal((9, 33)) * 3 + 1
+    ref = torch.nn.functional.layer_norm(torch.from_numpy(x), (33,), eps=1e-6).numpy()
+    np.testing.assert_allclose(O.layer_norm(x, 1e-6), ref, rtol=1e-12, atol=1e-12)
+    w, b = rng(3).standard_normal(33), rng(4).standard_normal(33)
+    ref = torch.nn.functional.layer_norm(torch.from_numpy(x), (33,), torch.from_numpy(w),
+                                         torch.from_numpy(b), eps=1e-6).numpy()
+    np.testing.assert_allclose(O.layer_norm(x, 1e-6, w, b), ref, rtol=1e-12, atol=1e-12)
+    # a constant row normalises to zero, so adaLN returns the shift
+    shift, scale = rng(5).standard_normal(33), rng(6).standard_normal(33)
+    np.testing.assert_allclose(O.adaln(np.full((2, 33), 4.25), shift, scale, 1e-6),
+                               np.tile(shift, (2, 1)), atol=1e-12)
+    y = O.layer_norm(x, 0.0)
+    np.testing.assert_allclose(y.mean(-1), 0, atol=1e-12)
+    np.testing.assert_allclose((y ** 2).mean(-1), 1, atol=1e-12)
+
+
+def test_rms_norm_closed_forms():
+    a = 2.5
+    signs = rng(7).choice([-1.0, 1.0], size=(4, 16))
+    g = 1 + 0.1 * rng(8).standard_normal(16)
+    keep = np.ones(16)
+    y = O.rms_norm(a * signs, g, keep, 0.0, 0, 8)
+    np.testing.assert_allclose(y, signs * g, rtol=1e-14)
+    # pruned channels do not enter the statistic (mode 0) and come out zero
+    keep = np.array([1] * 8 + [0] * 8, dtype=np.float64)
+    x = a * signs
+    x2 = x.copy()
+    x2[:, 8:] = 1e3 * rng(9).standard_normal((4, 8))
+    y1, y2 = O.rms_norm(x, g, keep, 0.0, 0, 8), O.rms_norm(x2, g, keep, 0.0, 0, 8)
+    np.testing.assert_array_equal(y1, y2)
+    np.testing.assert_allclose(y1[:, :8], signs[:, :8] * g[:8], rtol=1e-14)
+    np.testing.assert_array_equal(y1[:, 8:], 0.0)
+    # mode 1: each head has its own statistic, so scaling one head changes nothing
+    x = rng(10).standard_normal((3, 16))
+    xs = x.copy()
+    xs[:, 8:] *= 17.0
+    np.testing.assert_allclose(O.rms_norm(x, g, np.ones(16), 0.0, 1, 8),
+                               O.rms_norm(xs, g, np.ones(16), 0.0, 1, 8), rtol=1e-13)
+    # ... while in mode 0 it does
+    assert not np.allclose(O.rms_norm(x, g, np.ones(16), 0.0, 0, 8)[:, :8],
+                           O.rms_norm(xs, g, np.ones(16), 0.0, 0, 8)[:, :8])
+
+
+@pytest.mark.parametrize("dh,bands", [(128, (22, 21, 21)), (64, (12, 10, 10))])
+def test_rope_band_sizes(dh, bands):
+    assert O.rope_pairs(dh) == bands
+    assert sum(bands) == dh // 2
+
+
+def test_rope_angles_explicit_values():
+    grid, dh, th = (3, 4, 5), 64, 10000.0
+    p_t, p_h, p_w = O.rope_pairs(dh)
+    ang = O.rope_angles(grid, dh, th)
+    tok = lambda f, y, w: (f * grid[1] + y) * grid[2] + w
+    assert np.all(ang[tok(0, 0, 0)] == 0)
+    # the first pair of each band turns by the position itself
+    assert ang[tok(2, 0, 0), 0] == 2.0
+    assert ang[tok(0, 3, 0), p_t] == 3.0
+    assert ang[tok(0, 0, 4), p_t + p_h] == 4.0
+    # pair j of the frame band turns by f * theta^(-j / p_t)
+    np.testing.assert_allclose(ang[tok(1, 0, 0), 5], th ** (-5 / p_t), rtol=1e-15)
+    np.testing.assert_allclose(ang[tok(0, 2, 0), p_t + 3], 2 * th ** (-3 / p_h), rtol=1e-15)
+    # a token that differs only in w shares the frame and height angles
+    a, b = ang[tok(1, 2, 0)], ang[tok(1, 2, 3)]
+    np.testing.assert_array_equal(a[:p_t + p_h], b[:p_t + p_h])
+    assert np.all(a[p_t + p_h + 1:] != b[p_t + p_h + 1:])
+
+
+def test_rope_equals_complex_multiplication_and_is_relative():
+    grid, dh = (2, 3, 4), 64
+    ang = O.rope_angles(grid, dh, 10000.0)
+    N = ang.shape[0]
+    x = rng(11).standard_normal((N, 2, dh))
+    y = O.apply_rope(x, ang)
+    z = (x[..., 0::2] + 1j * x[..., 1::2]) * np.exp(1j * ang)[:, None, :]
+    np.testing.assert_allclose(y[..., 0::2], z.real, atol=1e-13)
+    np.testing.assert_allclose(y[..., 1::2], z.imag, atol=1e-13)
+    np.testing.assert_allclose(np.linalg.norm(y, axis=-1), np.linalg.norm(x, axis=-1), rtol=1e-13)
+    # <R(p) q, R(p') k> = <q, R(p' - p) k> along one axis (width, here)
+    q, k = rng(12).standard_normal((1, 1, dh)), rng(13).standard_normal((1, 1, dh))
+    tok = lambda f, y_, w: (f * grid[1] + y_) * grid[2] + w
+    lhs = np.sum(O.apply_rope(q, ang[[tok(1, 1, 1)]]) * O.apply_rope(k, ang[[tok(1, 1, 3)]]))
+    rhs = np.sum(q * O.apply_rope(k, ang[[tok(0, 0, 2)]]))
+    np.testing.assert_allclose(lhs, rhs, rtol=1e-12)
+
+
+def _attention_brute(q, k, v):
+    n, h, dh = q.shape
+    m = k.shape[0]
+    out = np.zeros((n, h, v.shape[2]))
+    for j in range(h):
+        for i in range(n):
+            logits = [sum(q[i, j, c] * k[t, j, c] for c in range(dh)) / math.sqrt(dh)
+                      for t in range(m)]
+            mx = max(logits)
+            w = [math.exp(l - mx) for l in logits]
+            z = sum(w)
+            for c in range(v.shape[2]):
+                out[i, j, c] = sum(w[t] * v[t, j, c] for t in range(m)) / z
+    return out
+
+
+def test_attention_brute_force():
+    r = rng(14)
+    q, k, v = r.standard_normal((5, 2, 4)) * 2, r.standard_normal((7, 2, 4)), r.standard_normal((7, 2, 4))
+    np.testing.assert_allclose(O.attention(q, k, v), _attention_brute(q, k, v), rtol=1e-12, atol=1e-14)
+
+
+def test_attention_special_cases():
+    r = rng(15)
+    dh = 4
+    # identical keys -> uniform weights -> mean of V
+    q = r.standard_normal((3, 1, dh))
+    k = np.tile(r.standard_normal((1, 1, dh)), (6, 1, 1))
+    v = r.standard_normal((6, 1, dh))
+    np.testing.assert_allclose(O.attention(q, k, v)[:, 0], np.tile(v[:, 0].mean(0), (3, 1)), rtol=1e-13)
+    # logit gap of ln 2 after the 1/sqrt(dh) scale -> weights 2/3 and 1/3
+    q = np.zeros((1, 1, dh)); q[0, 0, 0] = 2 * math.log(2.0)
+    k = np.zeros((2, 1, dh)); k[0, 0, 0] = 1.0
+    v = np.zeros((2, 1, dh)); v[0, 0, 0] = 3.0; v[1, 0, 0] = 0.0
+    np.testing.assert_allclose(O.attention(q, k, v)[0, 0, 0], 2.0, rtol=1e-14)
+    # one dominant logit selects its value row
+    q = np.zeros((1, 1, dh)); q[0, 0, 1] = 2000.0
+    k = r.standard_normal((5, 1, dh)) * 0.01; k[3, 0, 1] = 1.0
+    v = r.standard_normal((5, 1, dh))
+    np.testing.assert_allclose(O.attention(q, k, v)[0, 0], v[3, 0], rtol=1e-12)
+
+
+def test_gelu_tanh_textbook():
+    x = np.linspace(-6, 6, 241)
+    g = O.gelu_tanh(x)
+    assert O.gelu_tanh(np.array([0.0]))[0] == 0.0
+    np.testing.assert_allclose(g - O.gelu_tanh(-x), x, atol=1e-14)
+    exact = np.array([v * 0.5 * (1 + math.erf(v / math.sqrt(2))) for v in x])
+    assert np.max(np.abs(g - exact)) < 1e-3
+    assert np.max(np.abs(g - exact)) > 1e-5        # it is the tanh form, not the erf form
+
+
+# --------------------------------------------------------------------------- the block
+
+def _problem(has_cross=0, mode=0, grid=(2, 4, 4), ctx_len=16, seed_tag=""):
+    cfg = synth.tiny(has_cross=has_cross, grid=grid, qk_norm_mode=mode)
+    cfg.ctx_len = ctx_len if has_cross else 0
+    sh, L, M, A = synth.make_problem(cfg, seed_tag)
+    return cfg, synth.widen(sh), synth.widen(L), M, synth.widen(A)
+
+
+@pytest.mark.parametrize("has_cross,mode", [(0, 0), (0, 1), (1, 0)])
+def test_masked_dense_equals_compacted(has_cross, mode):
+    """Eq. 2 + export (Sec. 3.2) + index tables (Sec. 4.3): same function."""
+    cfg, W, LW, M, X = _problem(has_cross, mode)
+    for s in range(4):
+        a, ia = O.block_forward_masked(cfg, W, LW[0], M, s, 0, X["x"], X["t_emb"][s],
+                                       X.get("ctx"), want=True)
+        b, ib = O.block_forward_compacted(cfg, W, LW[0], M, s, 0, X["x"], X["t_emb"][s],
+                                          X.get("ctx"), want=True)
+        np.testing.assert_allclose(a, b, rtol=0, atol=1e-12 * np.abs(a).max())
+        np.testing.assert_allclose(ia["x1"], ib["x1"], rtol=0, atol=1e-12 * np.abs(ia["x1"]).max())
+        # the pruned branch is not the identity
+        assert np.abs(a - X["x"]).max() > 1e-2
+
+
+def test_row_slice_equals_full():
+    cfg, W, LW, M, X = _problem(1, 0)
+    rows = np.array([0, 5, 17, 31])
+    full = O.block_forward_compacted(cfg, W, LW[0], M, 1, 0, X["x"], X["t_emb"][1], X["ctx"])
+    part = O.block_forward_compacted(cfg, W, LW[0], M, 1, 0, X["x"], X["t_emb"][1], X["ctx"], rows=rows)
+    np.testing.assert_allclose(part, full[rows], rtol=1e-13, atol=1e-13)
+    part = O.block_forward_masked(cfg, W, LW[0], M, 1, 0, X["x"], X["t_emb"][1], X["ctx"], rows=rows)
+    np.testing.assert_allclose(part, full[rows], rtol=1e-11, atol=1e-11)
+
+
+def test_keep_all_is_the_unpruned_block():
+    cfg, W, LW, M, X = _problem()
+    M1 = dict(M)
+    M1["head_gate"] = np.ones_like(M["head_gate"])
+    M1["ffn_gate"] = np.ones_like(M["ffn_gate"])
+    a, ia = O.block_forward_compacted(cfg, W, LW[0], M1, 3, 0, X["x"], X["t_emb"][3], want=True)
+    # mode-0 QK norm over all retained channels is then the full-row RMSNorm
+    q_raw = O.linear(ia["xm"], LW[0]["wq"], LW[0]["bq"])
+    full = q_raw / np.sqrt((q_raw ** 2).mean(-1, keepdims=True) + cfg.ln_eps) * LW[0]["gq"]
+    ang = O.rope_angles(cfg.grid, cfg.head_dim, cfg.rope_theta)
+    np.testing.assert_allclose(ia["q"], O.apply_rope(full.reshape(-1, 4, 64), ang), rtol=1e-12, atol=1e-12)
+    b = O.block_forward_masked(cfg, W, LW[0], M1, 3, 0, X["x"], X["t_emb"][3])
+    np.testing.assert_allclose(a, b, atol=1e-12)
+
+
+def test_empty_masks_reduce_to_bias_branches():
+    cfg, W, LW, M, X = _problem()
+    M0 = dict(M)
+    M0["head_gate"] = np.zeros_like(M["head_gate"])
+    M0["ffn_gate"] = np.zeros_like(M["ffn_gate"])
+    mod = O.modulation(W["w_t"], W["b_t"], LW[0]["e_mod"], X["t_emb"][0])
+    for fn in (O.block_forward_masked, O.block_forward_compacted):
+        out, it = fn(cfg, W, LW[0], M0, 0, 0, X["x"], X["t_emb"][0], want=True)
+        x1 = X["x"] + mod[2] * LW[0]["bo"]
+        np.testing.assert_allclose(it["x1"], x1, atol=1e-14)
+        np.testing.assert_allclose(out, x1 + mod[5] * LW[0]["b_down"], atol=1e-14)
+
+
+def test_block_gate_zero_is_identity():
+    cfg, W, LW, M, X = _problem()
+    Mb = dict(M)
+    Mb["block_gate"] = np.zeros_like(M["block_gate"])
+    for fn in (O.block_forward_masked, O.block_forward_compacted):
+        np.testing.assert_array_equal(fn(cfg, W, LW[0], Mb, 1, 0, X["x"], X["t_emb"][1]), X["x"])
+
+
+def test_modulation_vectors_land_where_read():
+    """Zeroing gate_a removes the attention branch; 1+scale_f = 0 makes xm2 = shift_f."""
+    cfg, W, LW, M, X = _problem()
+    t = X["t_emb"][2]
+    base = (W["w_t"] @ t + W["b_t"]).reshape(6, cfg.dim)
+    lw = dict(LW[0])
+    e = lw["e_mod"].copy()
+    e[2] = -base[2]
+    e[4] = -1.0 - base[4]
+    lw["e_mod"] = e
+    out, it = O.block_forward_compacted(cfg, W, lw, M, 2, 0, X["x"], t, want=True)
+    np.testing.assert_array_equal(it["x1"], X["x"])
+    np.testing.assert_allclose(it["xm2"], np.tile(base[3] + e[3], (cfg.n_tokens, 1)), atol=1e-12)
+
+
+# --------------------------------------------------------------------------- FLOPs
+
+@pytest.mark.parametrize("has_cross", [0, 1])
+def test_flop_closed_form_matches_executed_contractions(has_cross):
+    cfg, W, LW, M, X = _problem(has_cross)
+    for s in range(4):
+        c = O.MacCounter()
+        O.block_forward_compacted(cfg, W, LW[0], M, s, 0, X["x"], X["t_emb"][s], X.get("ctx"), counter=c)
+        idx = O.compact_indices(cfg, M, s, 0)
+        f = O.block_flops(cfg.n_tokens, cfg.dim, cfg.head_dim, len(idx["heads"]), len(idx["ffn_ch"]),
+                          len(idx["xheads"]) if has_cross else 0, cfg.ctx_len)
+        assert c.flops == f
+
+
+def test_flop_keep_reproduces_paper_cut():
+    """The 14B-shaped keep schedule removes the paper's 24% of per-step FLOPs."""
+    cfg = synth.wan14b()
+    f = [O.block_flops(cfg.n_tokens, cfg.dim, cfg.head_dim, cfg.heads_kept[s][0],
+                       8 * cfg.chunks_kept[s][0]) for s in range(4)]
+    mean_keep = np.mean(f) / f[0]
+    assert abs((1 - mean_keep) - GOLD["wan14b_per_step_flop_cut"]["value"]) < 0.01
+    assert mean_keep <= GOLD["stop_criterion_mean_flops"]["value"] + 0.02
+    # the paper's U-shaped 1.3B retention averages to its ~83% final checkpoint
+    assert abs(np.mean(GOLD["wan13b_step_retention"]["value"]) - GOLD["wan13b_final_flop_ratio"]["value"]) < 0.01
+    # closed-form dense 14B block: 38.1 TFLOP, attention the largest share
+    assert abs(f[0] - 3.8125e13) / 3.8125e13 < 1e-3
+
+
+def test_denoise_with_all_blocks_off_is_geometric():
+    cfg, W, LW, M, X = _problem()
+    Mb = dict(M)
+    Mb["block_gate"] = np.zeros_like(M["block_gate"])
+    out = O.denoise(cfg, W, LW, Mb, X["x"], X["t_emb"])
+    np.testing.assert_allclose(out, X["x"] * (1 + 1 / GOLD["n_steps"]["value"]) ** 4, rtol=1e-14)
+
+
+# --------------------------------------------------------------------------- input generator
+
+def test_bf16_rounding_matches_torch():
+    torch = pytest.importorskip("torch")
+    a = np.concatenate([rng(16).standard_normal(5000).astype(np.float32),
+                        np.array([1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -1.0 - 2 ** -8, 0.0], np.float32)])
+    ref = torch.from_numpy(a).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(synth.f32_to_bf16_bits(a), ref)
+
+
+def test_config_keep_counts():
+    c2, c3 = synth.wan13b(), synth.wan14b()
+    assert [c2.heads_kept[s][0] for s in range(4)] == [12, 10, 9, 8]
+    assert [8 * c2.chunks_kept[s][0] for s in range(4)] == [8960, 7616, 6720, 5824]
+    assert [c3.heads_kept[s][0] for s in range(4)] == [40, 32, 28, 22]
+    assert [8 * c3.chunks_kept[s][0] for s in range(4)] == [13824, 11056, 9680, 7600]
+    assert c3.n_tokens == 32760 and synth.sweep720(0.5).n_tokens == 75600
