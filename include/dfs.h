@@ -1,0 +1,168 @@
+/*
+ * dfs.h - C ABI of the GB300 (sm_103a) engine for step-specific pruned video-DiT blocks
+ * ("Dynamic-in-Few-Step": a few-step distilled DiT whose every denoising step keeps its
+ * own subset of attention heads and FFN hidden-channel chunks, Sec. 3.2 and Sec. 4.3).
+ *
+ * Conventions shared by every entry point
+ *   - Tensors are row-major.  bf16 means IEEE bfloat16 bit patterns (uint16_t storage).
+ *   - Linear weights are [out, in] (so every projection is y = x W^T + b).
+ *   - "device" pointers are CUDA global-memory addresses of the current device; "host"
+ *     pointers are ordinary CPU memory.  Nothing here takes or returns torch types.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).  All GPU
+ *     work is enqueued on it; no entry point synchronises except dfs_plan_create,
+ *     dfs_plan_sync and the *_host variants, which say so.
+ *   - Errors are returned as dfs_status and never thrown across the ABI; dfs_last_error()
+ *     gives a message for the calling thread.  On any error nothing is written to `out`.
+ *   - A plan may be used from one host thread at a time.
+ */
+#ifndef DFS_H_
+#define DFS_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct dfs_plan dfs_plan; /* opaque; owned by the library */
+
+typedef enum {
+  DFS_OK = 0,
+  DFS_EINVAL = 1,        /* bad argument, shape, mask or pointer                      */
+  DFS_ENOMEM = 2,        /* device or host allocation failed                          */
+  DFS_ECUDA = 3,         /* a CUDA runtime / driver call failed                       */
+  DFS_ETIMEOUT = 4,      /* a kernel's bounded wait expired; its results are invalid   */
+  DFS_EUNSUPPORTED = 5   /* valid request this build does not implement                */
+} dfs_status;
+
+/* Block shapes.  N = grid_t * grid_h * grid_w latent tokens (frame-major).
+ *   dim = n_heads * head_dim, head_dim in {64, 128}, ffn_dim % ffn_chunk == 0,
+ *   ffn_chunk = 8 (App. A), n_steps = 4 (Sec. 3.1; 1..8 accepted).
+ *   qk_norm_mode: 0 = QK RMSNorm over the retained q (k) channels of a token row,
+ *                 1 = over each head's head_dim channels.
+ *   has_cross = 1 adds text cross-attention over ctx_len context tokens (1..4096). */
+typedef struct {
+  int dim, n_heads, head_dim, ffn_dim, ffn_chunk, n_layers, n_steps;
+  int grid_t, grid_h, grid_w;
+  int ctx_len, has_cross;
+  float ln_eps;      /* LayerNorm / RMSNorm epsilon (1e-6)       */
+  float rope_theta;  /* 3D RoPE base (1e4)                       */
+  int qk_norm_mode;
+} dfs_config;
+
+/* One layer's full (unpruned) weights; bf16 DEVICE pointers, borrowed for the duration
+ * of dfs_plan_create only (the plan keeps its own compacted copies).
+ *   wq, wk, wv, wo [dim, dim]; bq, bk, bv, bo [dim]; gq, gk [dim] (QK RMSNorm scales);
+ *   w_up [ffn_dim, dim]; b_up [ffn_dim]; w_down [dim, ffn_dim]; b_down [dim];
+ *   e_mod [6, dim] per-layer adaLN table (rows shift_a, scale_a, gate_a, shift_f,
+ *   scale_f, gate_f).  Cross-attention (only read when has_cross): cwq..cwo [dim, dim],
+ *   cbq..cbo, cgq, cgk, cln_w, cln_b [dim]. */
+typedef struct {
+  const void *wq, *bq, *wk, *bk, *wv, *bv, *wo, *bo, *gq, *gk;
+  const void *w_up, *b_up, *w_down, *b_down, *e_mod;
+  const void *cwq, *cbq, *cwk, *cbk, *cwv, *cbv, *cwo, *cbo, *cgq, *cgk, *cln_w, *cln_b;
+} dfs_layer_weights;
+
+/* Binary gates of Sec. 3.2 (1 = retained), HOST pointers, borrowed during create:
+ *   block_gate [n_steps][n_layers], head_gate [n_steps][n_layers][n_heads],
+ *   xhead_gate [n_steps][n_layers][n_heads] or NULL (= all cross heads kept),
+ *   ffn_gate [n_steps][n_layers][ffn_dim / ffn_chunk].  Values must be 0 or 1. */
+typedef struct {
+  const uint8_t *block_gate, *head_gate, *xhead_gate, *ffn_gate;
+} dfs_masks;
+
+/* Builds a plan (Sec. 4.3: the union super-model plus the per-step index tables I_t).
+ * Validates every argument on the host before any CUDA call, builds the ascending
+ * retained head / chunk lists per (step, layer), gathers the retained weight slices
+ * into dense bf16 panels on the device (one compaction kernel per panel), copies the
+ * full bias / modulation vectors, precomputes the RoPE tables and, with has_cross,
+ * the context keys / values per (step, layer); allocates the workspace for N tokens.
+ *   w_t [6*dim, dim], b_t [6*dim]: shared adaLN linear (bf16 device, borrowed).
+ *   ctx [ctx_len, dim] bf16 device or NULL when has_cross == 0 (borrowed).
+ * Synchronises `stream` before returning.  On failure *out is NULL and everything
+ * allocated so far is freed.  Errors: DFS_EINVAL, DFS_ENOMEM, DFS_ECUDA. */
+dfs_status dfs_plan_create(const dfs_config* cfg, const dfs_layer_weights* layers /*[n_layers]*/,
+                           const void* w_t, const void* b_t, const dfs_masks* masks,
+                           const void* ctx, void* stream, dfs_plan** out);
+
+/* Forward of layer 0 at denoising step `step` (0-based; the paper's t_{step+1}).
+ * x, out: [N, dim] bf16 device, caller-owned, must not alias.  t_emb: [dim] bf16
+ * device.  Computes, with the step's compacted weights only:
+ *   mod = W_t t_emb + b_t + E_l; xm = LN(x)(1+scale_a)+shift_a; qkv = xm Wqkv_s^T + b;
+ *   QK RMSNorm + 3D RoPE; attention over the retained heads; x1 = x + gate_a (o Wo_s^T + bo);
+ *   [cross-attention]; xm2 = LN(x1)(1+scale_f)+shift_f; h = GELU(xm2 Wup_s^T + bup_s);
+ *   out = x1 + gate_f (h Wdown_s^T + b_down).   A block gated off copies x to out.
+ * Errors: DFS_EINVAL (null pointer, step/layer out of range, x == out), DFS_ECUDA. */
+dfs_status dfs_block_forward(dfs_plan* plan, int step, const void* x, const void* t_emb,
+                             void* out, void* stream);
+
+/* As dfs_block_forward for any layer of the plan. */
+dfs_status dfs_block_forward_layer(dfs_plan* plan, int step, int layer, const void* x,
+                                   const void* t_emb, void* out, void* stream);
+
+/* End-to-end variant of dfs_block_forward_layer on HOST buffers: copies x [N, dim] and
+ * t_emb [dim] (bf16, host; pinned memory gives full copy speed) to plan-owned device
+ * staging, runs the forward and copies the result back to `out` (host).  Synchronises
+ * `stream` before returning. */
+dfs_status dfs_block_forward_host(dfs_plan* plan, int step, int layer, const void* x_host,
+                                  const void* t_emb_host, void* out_host, void* stream);
+
+/* Few-step denoising loop (Sec. 3.1, Fig. 1(b) rollout): for s in 0..n_steps-1, run
+ * every layer with its step-s structure (block-gated layers skipped), then
+ * latents <- latents + (1/cfg.n_steps) * v with v the last layer's output.
+ * latents: [N, dim] bf16 device, in/out.  t_embs: [n_steps, dim] bf16 device. */
+dfs_status dfs_denoise(dfs_plan* plan, void* latents, int n_steps, const void* t_embs,
+                       void* stream);
+
+/* Test hooks ---------------------------------------------------------------------- */
+
+/* Index lists of I_t for (step, layer).  kind: 0 = retained head ids, 1 = retained FFN
+ * chunk ids, 2 = retained cross-attention head ids.  Writes *count ids (ascending) to
+ * `out` (host, may be NULL to query the count). */
+dfs_status dfs_plan_indices(const dfs_plan* plan, int step, int layer, int kind,
+                            int32_t* out, int* count);
+
+/* Device address and shape of a compacted panel (bf16, row-major, leading dim *ld in
+ * elements).  which: 0 Wqkv [3 h_s dh, dim], 1 bqkv [3 h_s dh], 2 gq [h_s dh],
+ * 3 gk [h_s dh], 4 Wo [dim, h_s dh], 5 W_up [f_s, dim], 6 b_up [f_s],
+ * 7 W_down [dim, f_s]; cross: 8 cWq [hc dh, dim], 9 cbq, 10 cWkv [2 hc dh, dim],
+ * 11 cbkv, 12 cgq, 13 cgk, 14 cWo [dim, hc dh].  A panel with zero rows or columns
+ * returns *dev == NULL. */
+dfs_status dfs_plan_panel(const dfs_plan* plan, int step, int layer, int which,
+                          const void** dev, int64_t* rows, int64_t* cols, int64_t* ld);
+
+/* Algorithmic FLOPs (2 per multiply-add) of one block forward at (step, layer). */
+dfs_status dfs_plan_flops(const dfs_plan* plan, int step, int layer, double* flops);
+
+/* Workspace buffers left by the last forward on this plan (for intermediate checks):
+ * which: 0 xm [N, dim] bf16 (holds xm2 after the FFN norm), 1 qk [N, 2 h_s dh] bf16
+ * (q | k after RMSNorm + RoPE), 2 vT [h_s dh, ld] bf16, 3 attn [N, h_s dh] bf16,
+ * 4 x1 [N, dim] fp32, 5 h [N, f_s] bf16, 6 mod [6, dim] fp32.  *dtype: 0 bf16, 1 fp32.
+ * Shapes refer to the (step, layer) of the last forward. */
+dfs_status dfs_plan_workspace(const dfs_plan* plan, int which, void** dev, int64_t* rows,
+                              int64_t* cols, int64_t* ld, int* dtype);
+
+/* Waits for `stream` and reports whether any kernel of this plan hit its bounded wait
+ * limit since the last call (DFS_ETIMEOUT) or a CUDA error occurred (DFS_ECUDA).
+ * Clears the plan's device error word. */
+dfs_status dfs_plan_sync(dfs_plan* plan, void* stream);
+
+/* Soft mask -> hard gate rules of Sec. 4.1, host only (no CUDA call).
+ * kind 0 = block: g = (m > 0); kind 1 = head: m holds unit_size entries per head and the
+ * head is kept iff their mean (computed in double) is > 0; kind 2 = FFN chunk: one
+ * scalar per chunk, g = (m > 0).  m: [n_rows][n_units * unit_size] floats (host),
+ * g: [n_rows][n_units] (host). */
+dfs_status dfs_gates_from_soft_masks(int kind, int n_rows, int n_units, int unit_size,
+                                     const float* m, uint8_t* g);
+
+/* Frees every device and host resource of the plan (NULL is a no-op).  Waits for the
+ * plan's outstanding work on the device first. */
+void dfs_plan_destroy(dfs_plan* plan);
+
+/* Thread-local message of the last error returned on this thread ("" if none). */
+const char* dfs_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DFS_H_ */

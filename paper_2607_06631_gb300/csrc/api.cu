@@ -1,0 +1,757 @@
+// Host side of the C ABI (include/dfs.h): plan construction (index tables I_t and
+// compacted per-step panels, Sec. 4.3), the per-step block forward, the few-step loop
+// and the test hooks.  All device work goes to the caller's stream.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/dfs.h"
+#include "kernels.cuh"
+
+using dfs::bf16;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+dfs_status fail(dfs_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+#define DFS_CK(expr)                                                                           \
+  do {                                                                                         \
+    cudaError_t e_ = (expr);                                                                   \
+    if (e_ != cudaSuccess) return fail(DFS_ECUDA, "%s failed: %s", #expr, cudaGetErrorString(e_)); \
+  } while (0)
+
+// ------------------------------------------------------------------ tensor maps
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2D bf16 map over a row-major [outer, inner] array with row pitch `ld` elements, a box
+// of box_inner x box_outer elements (box_inner * 2 = 128 B) and 128-byte swizzle;
+// out-of-range elements read as zero.
+bool make_map(CUtensorMap* m, const void* base, long long inner, long long outer, long long ld, int box_inner,
+              int box_outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || inner <= 0 || outer <= 0) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_outer)};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+long long round_up(long long v, long long m) { return (v + m - 1) / m * m; }
+
+}  // namespace
+
+// ------------------------------------------------------------------ plan
+
+struct Panel {
+  bf16* p = nullptr;
+  long long rows = 0, cols = 0, ld = 0;
+};
+
+struct StepLayer {
+  int h_s = 0, f_s = 0, hc = 0;
+  std::vector<int> heads, chunks, xheads;
+  Panel P[15];       // indexed like dfs_plan_panel's `which`
+  bf16* kc = nullptr;    // cross-attention context keys, normalised [ctx_len, hc dh]
+  bf16* vct = nullptr;   // cross-attention context values, transposed [hc dh, ctx_ld]
+  dfs::GemmArgs g_qkv, g_o, g_up, g_down, g_cq, g_co;
+  dfs::AttnArgs a_self, a_cross;
+  double flops = 0;
+};
+
+struct LayerConst {
+  bf16* bo = nullptr;
+  bf16* bdown = nullptr;
+  bf16* emod = nullptr;
+  bf16* cbo = nullptr;
+  float* cln_w = nullptr;
+  float* cln_b = nullptr;
+};
+
+struct dfs_plan {
+  dfs_config cfg;
+  int N = 0, T = 0, L = 0, num_sms = 0, device = 0;
+  std::vector<uint8_t> block_gate;
+  std::vector<StepLayer> sl;  // [T * L]
+  std::vector<LayerConst> lc;
+  bf16* w_t = nullptr;
+  bf16* b_t = nullptr;
+  dfs::RopeTables rope{};
+  float* mod = nullptr;       // [6, d] for the current layer
+  float* mod_base = nullptr;  // [T, 6, d] W_t t_emb + b_t per step (denoise)
+  bf16* xm = nullptr;
+  bf16* qk = nullptr;
+  bf16* vt = nullptr;
+  long long vt_ld = 0, ctx_ld = 0;
+  bf16* attn = nullptr;
+  float* x1 = nullptr;
+  bf16* h = nullptr;
+  bf16* qc = nullptr;
+  bf16* act[2] = {nullptr, nullptr};
+  bf16* stage_x = nullptr;
+  bf16* stage_out = nullptr;
+  bf16* stage_t = nullptr;
+  int* err = nullptr;
+  std::vector<void*> allocs;
+  int last_step = -1, last_layer = -1;
+  int fault_alloc = -1, n_alloc = 0;  // host-side fault injection (DFS_FAULT_ALLOC=n)
+};
+
+namespace {
+
+dfs_status dev_alloc(dfs_plan* P, void** out, size_t bytes) {
+  *out = nullptr;
+  ++P->n_alloc;
+  if (P->fault_alloc > 0 && P->n_alloc == P->fault_alloc)
+    return fail(DFS_ENOMEM, "injected allocation failure at allocation %d", P->n_alloc);
+  if (bytes == 0) return DFS_OK;
+  cudaError_t e = cudaMalloc(out, bytes);
+  if (e != cudaSuccess) {
+    *out = nullptr;
+    (void)cudaGetLastError();
+    return fail(DFS_ENOMEM, "cudaMalloc(%zu) failed: %s", bytes, cudaGetErrorString(e));
+  }
+  P->allocs.push_back(*out);
+  return DFS_OK;
+}
+
+template <typename T>
+dfs_status alloc_n(dfs_plan* P, T** out, long long n) {
+  return dev_alloc(P, reinterpret_cast<void**>(out), static_cast<size_t>(n) * sizeof(T));
+}
+
+void free_plan(dfs_plan* P) {
+  if (!P) return;
+  for (void* p : P->allocs) cudaFree(p);
+  delete P;
+}
+
+// ------------------------------------------------------------------ validation (host only)
+
+dfs_status validate(const dfs_config* c, const dfs_layer_weights* layers, const void* w_t, const void* b_t,
+                    const dfs_masks* m, const void* ctx, dfs_plan** out) {
+  if (!out) return fail(DFS_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (!c) return fail(DFS_EINVAL, "cfg is NULL");
+  if (c->head_dim != 64 && c->head_dim != 128) return fail(DFS_EINVAL, "head_dim must be 64 or 128");
+  if (c->n_heads < 1 || c->dim != c->n_heads * c->head_dim)
+    return fail(DFS_EINVAL, "dim (%d) must equal n_heads * head_dim", c->dim);
+  if (c->dim > 8192) return fail(DFS_EUNSUPPORTED, "dim > 8192");
+  if (c->ffn_chunk != 8) return fail(DFS_EINVAL, "ffn_chunk must be 8");
+  if (c->ffn_dim < 8 || c->ffn_dim % c->ffn_chunk != 0)
+    return fail(DFS_EINVAL, "ffn_dim (%d) must be a positive multiple of ffn_chunk", c->ffn_dim);
+  if (c->n_layers < 1 || c->n_layers > 4096) return fail(DFS_EINVAL, "n_layers out of range");
+  if (c->n_steps < 1 || c->n_steps > 8) return fail(DFS_EINVAL, "n_steps must be in 1..8");
+  if (c->grid_t < 1 || c->grid_h < 1 || c->grid_w < 1) return fail(DFS_EINVAL, "grid dims must be >= 1");
+  const long long N = static_cast<long long>(c->grid_t) * c->grid_h * c->grid_w;
+  if (N > (1LL << 22)) return fail(DFS_EUNSUPPORTED, "more than 2^22 tokens");
+  if (c->has_cross != 0 && c->has_cross != 1) return fail(DFS_EINVAL, "has_cross must be 0 or 1");
+  if (c->has_cross && (c->ctx_len < 1 || c->ctx_len > 4096 || c->ctx_len % 8 != 0))
+    return fail(DFS_EINVAL, "ctx_len must be a multiple of 8 in 8..4096");
+  if (c->has_cross && !ctx) return fail(DFS_EINVAL, "ctx is NULL with has_cross");
+  if (c->qk_norm_mode != 0 && c->qk_norm_mode != 1) return fail(DFS_EINVAL, "qk_norm_mode must be 0 or 1");
+  if (!(c->ln_eps > 0.f) || !(c->rope_theta > 1.f)) return fail(DFS_EINVAL, "ln_eps / rope_theta out of range");
+  if (!layers || !w_t || !b_t || !m) return fail(DFS_EINVAL, "NULL weights or masks");
+  for (int l = 0; l < c->n_layers; ++l) {
+    const dfs_layer_weights& w = layers[l];
+    const void* req[] = {w.wq, w.bq, w.wk, w.bk, w.wv, w.bv, w.wo, w.bo, w.gq, w.gk, w.w_up, w.b_up, w.w_down,
+                         w.b_down, w.e_mod};
+    for (const void* p : req)
+      if (!p) return fail(DFS_EINVAL, "layer %d: NULL weight pointer", l);
+    if (c->has_cross) {
+      const void* rc[] = {w.cwq, w.cbq, w.cwk, w.cbk, w.cwv, w.cbv, w.cwo, w.cbo, w.cgq, w.cgk, w.cln_w, w.cln_b};
+      for (const void* p : rc)
+        if (!p) return fail(DFS_EINVAL, "layer %d: NULL cross-attention weight pointer", l);
+    }
+  }
+  if (!m->block_gate || !m->head_gate || !m->ffn_gate) return fail(DFS_EINVAL, "NULL gate array");
+  const long long TL = static_cast<long long>(c->n_steps) * c->n_layers;
+  auto check01 = [](const uint8_t* g, long long n) {
+    for (long long i = 0; i < n; ++i)
+      if (g[i] > 1) return false;
+    return true;
+  };
+  if (!check01(m->block_gate, TL) || !check01(m->head_gate, TL * c->n_heads) ||
+      !check01(m->ffn_gate, TL * (c->ffn_dim / c->ffn_chunk)) ||
+      (m->xhead_gate && !check01(m->xhead_gate, TL * c->n_heads)))
+    return fail(DFS_EINVAL, "gate values must be 0 or 1");
+  return DFS_OK;
+}
+
+// ------------------------------------------------------------------ GEMM / attention args
+
+dfs::GemmArgs gemm_args(dfs_plan* P, const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, int mode,
+                        const bf16* bias) {
+  dfs::GemmArgs g;
+  memset(&g, 0, sizeof(g));
+  g.tma_a = a;
+  g.tma_b = b;
+  g.M = M; g.N = N; g.K = K;
+  g.mode = mode;
+  g.bias = bias;
+  g.split = N;
+  g.err = P->err;
+  return g;
+}
+
+dfs_status upload_ints(dfs_plan* P, const std::vector<int>& v, int** out, cudaStream_t st) {
+  *out = nullptr;
+  if (v.empty()) return DFS_OK;
+  dfs_status s = alloc_n(P, out, static_cast<long long>(v.size()));
+  if (s) return s;
+  DFS_CK(cudaMemcpyAsync(*out, v.data(), v.size() * sizeof(int), cudaMemcpyHostToDevice, st));
+  return DFS_OK;
+}
+
+// Builds the index lists, gathers the panels and prebuilds every kernel argument of
+// one (step, layer).
+dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& w, const dfs_masks* m,
+                            const void* ctx, cudaStream_t st, std::vector<std::vector<int>>& keep_alive) {
+  const dfs_config& c = P->cfg;
+  const int d = c.dim, H = c.n_heads, dh = c.head_dim, NC = c.ffn_dim / c.ffn_chunk;
+  StepLayer& S = P->sl[s * P->L + l];
+  const long long base = static_cast<long long>(s) * c.n_layers + l;
+  for (int h = 0; h < H; ++h)
+    if (m->head_gate[base * H + h]) S.heads.push_back(h);
+  for (int k = 0; k < NC; ++k)
+    if (m->ffn_gate[base * NC + k]) S.chunks.push_back(k);
+  if (c.has_cross)
+    for (int h = 0; h < H; ++h)
+      if (!m->xhead_gate || m->xhead_gate[base * H + h]) S.xheads.push_back(h);
+  S.h_s = static_cast<int>(S.heads.size());
+  S.f_s = static_cast<int>(S.chunks.size()) * c.ffn_chunk;
+  S.hc = static_cast<int>(S.xheads.size());
+  const int hd = S.h_s * dh, hcd = S.hc * dh, fs = S.f_s;
+  const int N = P->N;
+
+  // index lists: rows (one per channel) and 16-byte segments (8 channels each)
+  std::vector<int> qk_rows, qk_segs, ffn_rows, x_rows, x_segs;
+  for (int h : S.heads)
+    for (int j = 0; j < dh; ++j) qk_rows.push_back(h * dh + j);
+  for (int h : S.heads)
+    for (int j = 0; j < dh / 8; ++j) qk_segs.push_back(h * dh / 8 + j);
+  for (int k : S.chunks)
+    for (int j = 0; j < c.ffn_chunk; ++j) ffn_rows.push_back(k * c.ffn_chunk + j);
+  for (int h : S.xheads)
+    for (int j = 0; j < dh; ++j) x_rows.push_back(h * dh + j);
+  for (int h : S.xheads)
+    for (int j = 0; j < dh / 8; ++j) x_segs.push_back(h * dh / 8 + j);
+  int *d_qk_rows, *d_qk_segs, *d_ffn_rows, *d_chunks, *d_x_rows, *d_x_segs;
+  dfs_status e;
+  if ((e = upload_ints(P, qk_rows, &d_qk_rows, st)) || (e = upload_ints(P, qk_segs, &d_qk_segs, st)) ||
+      (e = upload_ints(P, ffn_rows, &d_ffn_rows, st)) || (e = upload_ints(P, S.chunks, &d_chunks, st)) ||
+      (e = upload_ints(P, x_rows, &d_x_rows, st)) || (e = upload_ints(P, x_segs, &d_x_segs, st)))
+    return e;
+  keep_alive.push_back(qk_rows);
+  keep_alive.push_back(qk_segs);
+  keep_alive.push_back(ffn_rows);
+  keep_alive.push_back(x_rows);
+  keep_alive.push_back(x_segs);
+
+  auto mk = [&](int which, long long rows, long long cols) -> dfs_status {
+    Panel& p = S.P[which];
+    p.rows = rows; p.cols = cols; p.ld = cols;
+    if (rows * cols == 0) return DFS_OK;
+    return alloc_n(P, &p.p, rows * cols);
+  };
+  const bf16* wq = static_cast<const bf16*>(w.wq);
+  const bf16* wk = static_cast<const bf16*>(w.wk);
+  const bf16* wv = static_cast<const bf16*>(w.wv);
+  if ((e = mk(0, 3LL * hd, d)) || (e = mk(1, 1, 3LL * hd)) || (e = mk(2, 1, hd)) || (e = mk(3, 1, hd)) ||
+      (e = mk(4, d, hd)) || (e = mk(5, fs, d)) || (e = mk(6, 1, fs)) || (e = mk(7, d, fs)))
+    return e;
+  if (c.has_cross) {
+    if ((e = mk(8, hcd, d)) || (e = mk(9, 1, hcd)) || (e = mk(10, 2LL * hcd, d)) || (e = mk(11, 1, 2LL * hcd)) ||
+        (e = mk(12, 1, hcd)) || (e = mk(13, 1, hcd)) || (e = mk(14, d, hcd)))
+      return e;
+  }
+  // K1 gathers
+  if (hd > 0) {
+    bf16* Wqkv = S.P[0].p;
+    DFS_CK(dfs::launch_gather_rows(Wqkv, d, wq, d, d_qk_rows, hd, d, st));
+    DFS_CK(dfs::launch_gather_rows(Wqkv + static_cast<long long>(hd) * d, d, wk, d, d_qk_rows, hd, d, st));
+    DFS_CK(dfs::launch_gather_rows(Wqkv + 2LL * hd * d, d, wv, d, d_qk_rows, hd, d, st));
+    bf16* b = S.P[1].p;
+    DFS_CK(dfs::launch_gather_segs(b, 0, static_cast<const bf16*>(w.bq), 0, d_qk_segs, hd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_segs(b + hd, 0, static_cast<const bf16*>(w.bk), 0, d_qk_segs, hd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_segs(b + 2 * hd, 0, static_cast<const bf16*>(w.bv), 0, d_qk_segs, hd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[2].p, 0, static_cast<const bf16*>(w.gq), 0, d_qk_segs, hd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[3].p, 0, static_cast<const bf16*>(w.gk), 0, d_qk_segs, hd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[4].p, hd, static_cast<const bf16*>(w.wo), d, d_qk_segs, hd / 8, d, st));
+  }
+  if (fs > 0) {
+    const int nch = static_cast<int>(S.chunks.size());
+    DFS_CK(dfs::launch_gather_rows(S.P[5].p, d, static_cast<const bf16*>(w.w_up), d, d_ffn_rows, fs, d, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[6].p, 0, static_cast<const bf16*>(w.b_up), 0, d_chunks, nch, 1, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[7].p, fs, static_cast<const bf16*>(w.w_down), c.ffn_dim, d_chunks, nch, d,
+                                   st));
+  }
+  if (c.has_cross && hcd > 0) {
+    DFS_CK(dfs::launch_gather_rows(S.P[8].p, d, static_cast<const bf16*>(w.cwq), d, d_x_rows, hcd, d, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[9].p, 0, static_cast<const bf16*>(w.cbq), 0, d_x_segs, hcd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_rows(S.P[10].p, d, static_cast<const bf16*>(w.cwk), d, d_x_rows, hcd, d, st));
+    DFS_CK(dfs::launch_gather_rows(S.P[10].p + static_cast<long long>(hcd) * d, d,
+                                   static_cast<const bf16*>(w.cwv), d, d_x_rows, hcd, d, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[11].p, 0, static_cast<const bf16*>(w.cbk), 0, d_x_segs, hcd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[11].p + hcd, 0, static_cast<const bf16*>(w.cbv), 0, d_x_segs, hcd / 8, 1,
+                                   st));
+    DFS_CK(dfs::launch_gather_segs(S.P[12].p, 0, static_cast<const bf16*>(w.cgq), 0, d_x_segs, hcd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[13].p, 0, static_cast<const bf16*>(w.cgk), 0, d_x_segs, hcd / 8, 1, st));
+    DFS_CK(dfs::launch_gather_segs(S.P[14].p, hcd, static_cast<const bf16*>(w.cwo), d, d_x_segs, hcd / 8, d,
+                                   st));
+  }
+
+  // kernel arguments
+  const LayerConst& C = P->lc[l];
+  CUtensorMap ma, mb;
+  const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(dh)));
+  if (hd > 0) {
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[0].p, d, 3LL * hd, d, 64, 256))
+      return fail(DFS_ECUDA, "tensor map (QKV) failed");
+    S.g_qkv = gemm_args(P, ma, mb, N, 3 * hd, d, dfs::kEpiBias, S.P[1].p);
+    S.g_qkv.out = P->qk; S.g_qkv.ldo = 2 * hd; S.g_qkv.split = 2 * hd;
+    S.g_qkv.out_t = P->vt; S.g_qkv.ldt = P->vt_ld;
+    if (!make_map(&ma, P->attn, hd, N, hd, 64, 128) || !make_map(&mb, S.P[4].p, hd, d, hd, 64, 256))
+      return fail(DFS_ECUDA, "tensor map (O) failed");
+    S.g_o = gemm_args(P, ma, mb, N, d, hd, dfs::kEpiGatedRes, C.bo);
+    S.g_o.out = P->x1; S.g_o.ldo = d; S.g_o.out_f32 = 1; S.g_o.ldr = d; S.g_o.res_f32 = 0;
+    dfs::AttnArgs& A = S.a_self;
+    memset(&A, 0, sizeof(A));
+    if (!make_map(&A.tma_q, P->qk, 2LL * hd, N, 2LL * hd, 64, 128) ||
+        !make_map(&A.tma_vt, P->vt, N, hd, P->vt_ld, 64, dh))
+      return fail(DFS_ECUDA, "tensor map (attention) failed");
+    A.tma_k = A.tma_q;
+    A.n_q = N; A.n_kv = N; A.n_heads = S.h_s; A.q_col0 = 0; A.k_col0 = hd;
+    A.out = P->attn; A.ldo = hd; A.scale_log2 = scale_log2; A.err = P->err;
+  }
+  if (fs > 0) {
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[5].p, d, fs, d, 64, 256))
+      return fail(DFS_ECUDA, "tensor map (up) failed");
+    S.g_up = gemm_args(P, ma, mb, N, fs, d, dfs::kEpiBiasGelu, S.P[6].p);
+    S.g_up.out = P->h; S.g_up.ldo = fs;
+    if (!make_map(&ma, P->h, fs, N, fs, 64, 128) || !make_map(&mb, S.P[7].p, fs, d, fs, 64, 256))
+      return fail(DFS_ECUDA, "tensor map (down) failed");
+    S.g_down = gemm_args(P, ma, mb, N, d, fs, dfs::kEpiGatedRes, C.bdown);
+    S.g_down.ldo = d; S.g_down.out_f32 = 0; S.g_down.res = P->x1; S.g_down.ldr = d; S.g_down.res_f32 = 1;
+  }
+  if (c.has_cross && hcd > 0) {
+    // context keys / values of this step's cross heads, once per plan
+    if ((e = alloc_n(P, &S.kc, static_cast<long long>(c.ctx_len) * hcd)) ||
+        (e = alloc_n(P, &S.vct, static_cast<long long>(hcd) * P->ctx_ld)))
+      return e;
+    if (!make_map(&ma, ctx, d, c.ctx_len, d, 64, 128) || !make_map(&mb, S.P[10].p, d, 2LL * hcd, d, 64, 256))
+      return fail(DFS_ECUDA, "tensor map (cross kv) failed");
+    dfs::GemmArgs kv = gemm_args(P, ma, mb, c.ctx_len, 2 * hcd, d, dfs::kEpiBias, S.P[11].p);
+    kv.out = S.kc; kv.ldo = hcd; kv.split = hcd; kv.out_t = S.vct; kv.ldt = P->ctx_ld;
+    DFS_CK(dfs::launch_gemm(kv, P->num_sms, st));
+    DFS_CK(dfs::launch_qk_norm_rope(S.kc, hcd, c.ctx_len, 0, hcd, nullptr, S.P[13].p, dh, c.qk_norm_mode,
+                                    c.ln_eps, nullptr, st));
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[8].p, d, hcd, d, 64, 256))
+      return fail(DFS_ECUDA, "tensor map (cross q) failed");
+    S.g_cq = gemm_args(P, ma, mb, N, hcd, d, dfs::kEpiBias, S.P[9].p);
+    S.g_cq.out = P->qc; S.g_cq.ldo = hcd;
+    if (!make_map(&ma, P->attn, hcd, N, hcd, 64, 128) || !make_map(&mb, S.P[14].p, hcd, d, hcd, 64, 256))
+      return fail(DFS_ECUDA, "tensor map (cross o) failed");
+    S.g_co = gemm_args(P, ma, mb, N, d, hcd, dfs::kEpiGatedRes, C.cbo);
+    S.g_co.out = P->x1; S.g_co.ldo = d; S.g_co.out_f32 = 1; S.g_co.res = P->x1; S.g_co.ldr = d;
+    S.g_co.res_f32 = 1; S.g_co.gate = nullptr;
+    dfs::AttnArgs& A = S.a_cross;
+    memset(&A, 0, sizeof(A));
+    if (!make_map(&A.tma_q, P->qc, hcd, N, hcd, 64, 128) || !make_map(&A.tma_k, S.kc, hcd, c.ctx_len, hcd, 64, 128) ||
+        !make_map(&A.tma_vt, S.vct, c.ctx_len, hcd, P->ctx_ld, 64, dh))
+      return fail(DFS_ECUDA, "tensor map (cross attention) failed");
+    A.n_q = N; A.n_kv = c.ctx_len; A.n_heads = S.hc; A.q_col0 = 0; A.k_col0 = 0;
+    A.out = P->attn; A.ldo = hcd; A.scale_log2 = scale_log2; A.err = P->err;
+  }
+  const double Nd = N, dd = d;
+  S.flops = 8 * Nd * dd * dh * S.h_s + 4 * Nd * Nd * dh * S.h_s + 4 * Nd * dd * S.f_s;
+  if (c.has_cross)
+    S.flops += 4 * Nd * dd * dh * S.hc + 4.0 * c.ctx_len * dd * dh * S.hc + 4 * Nd * c.ctx_len * dh * S.hc;
+  return DFS_OK;
+}
+
+dfs_status create_impl(dfs_plan* P, const dfs_layer_weights* layers, const void* w_t, const void* b_t,
+                       const dfs_masks* m, const void* ctx, cudaStream_t st) {
+  const dfs_config& c = P->cfg;
+  const int d = c.dim, dh = c.head_dim;
+  DFS_CK(cudaGetDevice(&P->device));
+  DFS_CK(cudaDeviceGetAttribute(&P->num_sms, cudaDevAttrMultiProcessorCount, P->device));
+  if (!encode_fn()) return fail(DFS_ECUDA, "cuTensorMapEncodeTiled is unavailable");
+  DFS_CK(dfs::gemm_prepare());
+  DFS_CK(dfs::attention_prepare());
+  const long long N = P->N;
+  dfs_status e;
+  if ((e = alloc_n(P, &P->err, 1))) return e;
+  DFS_CK(cudaMemsetAsync(P->err, 0, sizeof(int), st));
+
+  // shared adaLN linear and per-layer constants
+  if ((e = alloc_n(P, &P->w_t, 6LL * d * d)) || (e = alloc_n(P, &P->b_t, 6LL * d))) return e;
+  DFS_CK(cudaMemcpyAsync(P->w_t, w_t, 12LL * d * d, cudaMemcpyDeviceToDevice, st));
+  DFS_CK(cudaMemcpyAsync(P->b_t, b_t, 12LL * d, cudaMemcpyDeviceToDevice, st));
+  P->lc.resize(P->L);
+  for (int l = 0; l < P->L; ++l) {
+    LayerConst& C = P->lc[l];
+    if ((e = alloc_n(P, &C.bo, d)) || (e = alloc_n(P, &C.bdown, d)) || (e = alloc_n(P, &C.emod, 6LL * d)))
+      return e;
+    DFS_CK(cudaMemcpyAsync(C.bo, layers[l].bo, 2LL * d, cudaMemcpyDeviceToDevice, st));
+    DFS_CK(cudaMemcpyAsync(C.bdown, layers[l].b_down, 2LL * d, cudaMemcpyDeviceToDevice, st));
+    DFS_CK(cudaMemcpyAsync(C.emod, layers[l].e_mod, 12LL * d, cudaMemcpyDeviceToDevice, st));
+    if (c.has_cross) {
+      if ((e = alloc_n(P, &C.cbo, d)) || (e = alloc_n(P, &C.cln_w, d)) || (e = alloc_n(P, &C.cln_b, d))) return e;
+      DFS_CK(cudaMemcpyAsync(C.cbo, layers[l].cbo, 2LL * d, cudaMemcpyDeviceToDevice, st));
+      DFS_CK(dfs::launch_to_f32(C.cln_w, static_cast<const bf16*>(layers[l].cln_w), d, st));
+      DFS_CK(dfs::launch_to_f32(C.cln_b, static_cast<const bf16*>(layers[l].cln_b), d, st));
+    }
+  }
+
+  // 3D RoPE tables (angles in double, stored fp32)
+  {
+    const int half = dh / 2, p_hw = dh / 6, p_t = half - 2 * p_hw;
+    const int G[3] = {c.grid_t, c.grid_h, c.grid_w};
+    const int Pn[3] = {p_t, p_hw, p_hw};
+    std::vector<float> host;
+    size_t off[6];
+    for (int a = 0; a < 3; ++a) {
+      off[2 * a] = host.size();
+      for (int pos = 0; pos < G[a]; ++pos)
+        for (int j = 0; j < Pn[a]; ++j)
+          host.push_back(static_cast<float>(std::cos(pos * std::pow(static_cast<double>(c.rope_theta),
+                                                                    -static_cast<double>(j) / Pn[a]))));
+      off[2 * a + 1] = host.size();
+      for (int pos = 0; pos < G[a]; ++pos)
+        for (int j = 0; j < Pn[a]; ++j)
+          host.push_back(static_cast<float>(std::sin(pos * std::pow(static_cast<double>(c.rope_theta),
+                                                                    -static_cast<double>(j) / Pn[a]))));
+    }
+    float* t;
+    if ((e = alloc_n(P, &t, static_cast<long long>(host.size())))) return e;
+    DFS_CK(cudaMemcpy(t, host.data(), host.size() * sizeof(float), cudaMemcpyHostToDevice));
+    P->rope.cos_t = t + off[0]; P->rope.sin_t = t + off[1];
+    P->rope.cos_h = t + off[2]; P->rope.sin_h = t + off[3];
+    P->rope.cos_w = t + off[4]; P->rope.sin_w = t + off[5];
+    P->rope.grid_h = c.grid_h; P->rope.grid_w = c.grid_w;
+    P->rope.p_t = p_t; P->rope.p_h = p_hw; P->rope.p_w = p_hw;
+  }
+
+  // workspace for N tokens, sized by the largest step structure
+  int hmax = 0, fmax = 0, hcmax = 0;
+  {
+    const int H = c.n_heads, NC = c.ffn_dim / c.ffn_chunk;
+    for (long long i = 0; i < static_cast<long long>(P->T) * P->L; ++i) {
+      int hs = 0, ch = 0, xh = 0;
+      for (int h = 0; h < H; ++h) hs += m->head_gate[i * H + h];
+      for (int k = 0; k < NC; ++k) ch += m->ffn_gate[i * NC + k];
+      if (c.has_cross)
+        for (int h = 0; h < H; ++h) xh += m->xhead_gate ? m->xhead_gate[i * H + h] : 1;
+      hmax = std::max(hmax, hs);
+      fmax = std::max(fmax, ch * c.ffn_chunk);
+      hcmax = std::max(hcmax, xh);
+    }
+  }
+  P->vt_ld = round_up(N, 64);
+  P->ctx_ld = round_up(c.has_cross ? c.ctx_len : 8, 64);
+  const long long amax = static_cast<long long>(std::max(hmax, hcmax)) * dh;
+  if ((e = alloc_n(P, &P->mod, 6LL * d)) || (e = alloc_n(P, &P->mod_base, 6LL * d * P->T)) ||
+      (e = alloc_n(P, &P->xm, N * d)) || (e = alloc_n(P, &P->qk, N * 2 * hmax * dh)) ||
+      (e = alloc_n(P, &P->vt, static_cast<long long>(hmax) * dh * P->vt_ld)) || (e = alloc_n(P, &P->attn, N * amax)) ||
+      (e = alloc_n(P, &P->x1, N * d)) || (e = alloc_n(P, &P->h, N * fmax)) ||
+      (e = alloc_n(P, &P->qc, N * static_cast<long long>(hcmax) * dh)) || (e = alloc_n(P, &P->act[0], N * d)) ||
+      (e = alloc_n(P, &P->act[1], N * d)) || (e = alloc_n(P, &P->stage_x, N * d)) ||
+      (e = alloc_n(P, &P->stage_out, N * d)) || (e = alloc_n(P, &P->stage_t, d)))
+    return e;
+  if (hmax > 0) DFS_CK(cudaMemsetAsync(P->vt, 0, sizeof(bf16) * hmax * dh * P->vt_ld, st));
+
+  // per (step, layer): index tables, compacted panels, kernel arguments
+  std::vector<std::vector<int>> keep_alive;  // host index lists stay valid until the sync below
+  P->sl.resize(static_cast<size_t>(P->T) * P->L);
+  for (int s = 0; s < P->T; ++s)
+    for (int l = 0; l < P->L; ++l)
+      if ((e = build_step_layer(P, s, l, layers[l], m, ctx, st, keep_alive))) return e;
+  DFS_CK(cudaStreamSynchronize(st));
+  int herr = 0;
+  DFS_CK(cudaMemcpy(&herr, P->err, sizeof(int), cudaMemcpyDeviceToHost));
+  if (herr) return fail(DFS_ETIMEOUT, "a kernel gave up waiting during plan creation");
+  return DFS_OK;
+}
+
+// ------------------------------------------------------------------ forward
+
+dfs_status forward_impl(dfs_plan* P, int s, int l, const bf16* x, bf16* out, cudaStream_t st) {
+  // P->mod holds this layer's six modulation vectors
+  const dfs_config& c = P->cfg;
+  const int d = c.dim, dh = c.head_dim;
+  const int N = P->N;
+  StepLayer& S = P->sl[s * P->L + l];
+  const LayerConst& C = P->lc[l];
+  const float* shift_a = P->mod;
+  const float* scale_a = P->mod + d;
+  const float* gate_a = P->mod + 2 * d;
+  const float* shift_f = P->mod + 3 * d;
+  const float* scale_f = P->mod + 4 * d;
+  const float* gate_f = P->mod + 5 * d;
+  P->last_step = s;
+  P->last_layer = l;
+
+  DFS_CK(dfs::launch_row_norm(P->xm, x, 0, N, d, scale_a, 1.f, shift_a, c.ln_eps, st));
+  if (S.h_s > 0) {
+    const int hd = S.h_s * dh;
+    DFS_CK(dfs::launch_gemm(S.g_qkv, P->num_sms, st));
+    DFS_CK(dfs::launch_qk_norm_rope(P->qk, 2LL * hd, N, hd, hd, S.P[2].p, S.P[3].p, dh, c.qk_norm_mode, c.ln_eps,
+                                    &P->rope, st));
+    DFS_CK(dfs::launch_attention(S.a_self, dh, st));
+    dfs::GemmArgs g = S.g_o;
+    g.res = x;
+    g.gate = gate_a;
+    DFS_CK(dfs::launch_gemm(g, P->num_sms, st));
+  } else {
+    DFS_CK(dfs::launch_bias_residual(P->x1, 1, x, 0, gate_a, C.bo, N, d, st));
+  }
+  if (c.has_cross) {
+    DFS_CK(dfs::launch_row_norm(P->xm, P->x1, 1, N, d, C.cln_w, 0.f, C.cln_b, c.ln_eps, st));
+    if (S.hc > 0) {
+      const int hcd = S.hc * dh;
+      DFS_CK(dfs::launch_gemm(S.g_cq, P->num_sms, st));
+      DFS_CK(dfs::launch_qk_norm_rope(P->qc, hcd, N, hcd, 0, S.P[12].p, nullptr, dh, c.qk_norm_mode, c.ln_eps,
+                                      nullptr, st));
+      DFS_CK(dfs::launch_attention(S.a_cross, dh, st));
+      DFS_CK(dfs::launch_gemm(S.g_co, P->num_sms, st));
+    } else {
+      DFS_CK(dfs::launch_bias_residual(P->x1, 1, P->x1, 1, nullptr, C.cbo, N, d, st));
+    }
+  }
+  DFS_CK(dfs::launch_row_norm(P->xm, P->x1, 1, N, d, scale_f, 1.f, shift_f, c.ln_eps, st));
+  if (S.f_s > 0) {
+    DFS_CK(dfs::launch_gemm(S.g_up, P->num_sms, st));
+    dfs::GemmArgs g = S.g_down;
+    g.out = out;
+    g.gate = gate_f;
+    DFS_CK(dfs::launch_gemm(g, P->num_sms, st));
+  } else {
+    DFS_CK(dfs::launch_bias_residual(out, 0, P->x1, 1, gate_f, C.bdown, N, d, st));
+  }
+  return DFS_OK;
+}
+
+dfs_status check_forward_args(dfs_plan* P, int step, int layer, const void* x, const void* t_emb, void* out) {
+  if (!P) return fail(DFS_EINVAL, "plan is NULL");
+  if (!x || !t_emb || !out) return fail(DFS_EINVAL, "NULL x, t_emb or out");
+  if (x == out) return fail(DFS_EINVAL, "x and out must not alias");
+  if (step < 0 || step >= P->T) return fail(DFS_EINVAL, "step %d out of range [0, %d)", step, P->T);
+  if (layer < 0 || layer >= P->L) return fail(DFS_EINVAL, "layer %d out of range [0, %d)", layer, P->L);
+  return DFS_OK;
+}
+
+dfs_status block_layer(dfs_plan* P, int step, int layer, const bf16* x, const bf16* t_emb, bf16* out,
+                       cudaStream_t st) {
+  const int d = P->cfg.dim;
+  if (!P->block_gate[static_cast<size_t>(step) * P->L + layer]) {
+    DFS_CK(cudaMemcpyAsync(out, x, sizeof(bf16) * P->N * d, cudaMemcpyDeviceToDevice, st));
+    return DFS_OK;
+  }
+  DFS_CK(dfs::launch_modulation(P->mod, P->w_t, P->b_t, P->lc[layer].emod, t_emb, 6 * d, d, st));
+  return forward_impl(P, step, layer, x, out, st);
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ C ABI
+
+extern "C" {
+
+dfs_status dfs_plan_create(const dfs_config* cfg, const dfs_layer_weights* layers, const void* w_t,
+                           const void* b_t, const dfs_masks* masks, const void* ctx, void* stream, dfs_plan** out) {
+  g_last_error.clear();
+  dfs_status e = validate(cfg, layers, w_t, b_t, masks, ctx, out);
+  if (e) return e;
+  dfs_plan* P = new (std::nothrow) dfs_plan();
+  if (!P) return fail(DFS_ENOMEM, "host allocation failed");
+  P->cfg = *cfg;
+  P->T = cfg->n_steps;
+  P->L = cfg->n_layers;
+  P->N = cfg->grid_t * cfg->grid_h * cfg->grid_w;
+  P->block_gate.assign(masks->block_gate, masks->block_gate + static_cast<size_t>(P->T) * P->L);
+  if (const char* f = getenv("DFS_FAULT_ALLOC")) P->fault_alloc = atoi(f);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  e = create_impl(P, layers, w_t, b_t, masks, ctx, st);
+  if (e) {
+    cudaStreamSynchronize(st);
+    (void)cudaGetLastError();
+    free_plan(P);
+    return e;
+  }
+  *out = P;
+  return DFS_OK;
+}
+
+dfs_status dfs_block_forward_layer(dfs_plan* plan, int step, int layer, const void* x, const void* t_emb,
+                                   void* out, void* stream) {
+  dfs_status e = check_forward_args(plan, step, layer, x, t_emb, out);
+  if (e) return e;
+  return block_layer(plan, step, layer, static_cast<const bf16*>(x), static_cast<const bf16*>(t_emb),
+                     static_cast<bf16*>(out), static_cast<cudaStream_t>(stream));
+}
+
+dfs_status dfs_block_forward(dfs_plan* plan, int step, const void* x, const void* t_emb, void* out, void* stream) {
+  return dfs_block_forward_layer(plan, step, 0, x, t_emb, out, stream);
+}
+
+dfs_status dfs_block_forward_host(dfs_plan* plan, int step, int layer, const void* x_host, const void* t_emb_host,
+                                  void* out_host, void* stream) {
+  dfs_status e = check_forward_args(plan, step, layer, x_host, t_emb_host, out_host);
+  if (e) return e;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t bytes = sizeof(bf16) * plan->N * plan->cfg.dim;
+  DFS_CK(cudaMemcpyAsync(plan->stage_x, x_host, bytes, cudaMemcpyHostToDevice, st));
+  DFS_CK(cudaMemcpyAsync(plan->stage_t, t_emb_host, sizeof(bf16) * plan->cfg.dim, cudaMemcpyHostToDevice, st));
+  e = block_layer(plan, step, layer, plan->stage_x, plan->stage_t, plan->stage_out, st);
+  if (e) return e;
+  DFS_CK(cudaMemcpyAsync(out_host, plan->stage_out, bytes, cudaMemcpyDeviceToHost, st));
+  DFS_CK(cudaStreamSynchronize(st));
+  return DFS_OK;
+}
+
+dfs_status dfs_denoise(dfs_plan* P, void* latents, int n_steps, const void* t_embs, void* stream) {
+  if (!P || !latents || !t_embs) return fail(DFS_EINVAL, "NULL plan, latents or t_embs");
+  if (n_steps < 1 || n_steps > P->T) return fail(DFS_EINVAL, "n_steps must be in 1..%d", P->T);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int d = P->cfg.dim;
+  bf16* lat = static_cast<bf16*>(latents);
+  const bf16* temb = static_cast<const bf16*>(t_embs);
+  for (int s = 0; s < n_steps; ++s) {
+    float* base = P->mod_base + 6LL * d * s;
+    DFS_CK(dfs::launch_modulation(base, P->w_t, P->b_t, nullptr, temb + static_cast<long long>(s) * d, 6 * d, d, st));
+    const bf16* cur = lat;
+    int ping = 0;
+    for (int l = 0; l < P->L; ++l) {
+      if (!P->block_gate[static_cast<size_t>(s) * P->L + l]) continue;
+      DFS_CK(dfs::launch_add_table(P->mod, base, P->lc[l].emod, 6 * d, st));
+      bf16* dst = P->act[ping];
+      dfs_status e = forward_impl(P, s, l, cur, dst, st);
+      if (e) return e;
+      cur = dst;
+      ping ^= 1;
+    }
+    DFS_CK(dfs::launch_euler(lat, cur, 1.f / P->cfg.n_steps, static_cast<long long>(P->N) * d, st));
+  }
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_indices(const dfs_plan* P, int step, int layer, int kind, int32_t* out, int* count) {
+  if (!P || !count) return fail(DFS_EINVAL, "NULL plan or count");
+  if (step < 0 || step >= P->T || layer < 0 || layer >= P->L) return fail(DFS_EINVAL, "step/layer out of range");
+  const StepLayer& S = P->sl[step * P->L + layer];
+  const std::vector<int>* v = kind == 0 ? &S.heads : kind == 1 ? &S.chunks : kind == 2 ? &S.xheads : nullptr;
+  if (!v) return fail(DFS_EINVAL, "kind must be 0, 1 or 2");
+  *count = static_cast<int>(v->size());
+  if (out)
+    for (size_t i = 0; i < v->size(); ++i) out[i] = (*v)[i];
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_panel(const dfs_plan* P, int step, int layer, int which, const void** dev, int64_t* rows,
+                          int64_t* cols, int64_t* ld) {
+  if (!P || !dev || !rows || !cols || !ld) return fail(DFS_EINVAL, "NULL argument");
+  if (step < 0 || step >= P->T || layer < 0 || layer >= P->L) return fail(DFS_EINVAL, "step/layer out of range");
+  if (which < 0 || which > 14 || (which > 7 && !P->cfg.has_cross)) return fail(DFS_EINVAL, "bad panel id");
+  const Panel& p = P->sl[step * P->L + layer].P[which];
+  *dev = p.p; *rows = p.rows; *cols = p.cols; *ld = p.ld;
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_flops(const dfs_plan* P, int step, int layer, double* flops) {
+  if (!P || !flops) return fail(DFS_EINVAL, "NULL argument");
+  if (step < 0 || step >= P->T || layer < 0 || layer >= P->L) return fail(DFS_EINVAL, "step/layer out of range");
+  *flops = P->block_gate[static_cast<size_t>(step) * P->L + layer] ? P->sl[step * P->L + layer].flops : 0.0;
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_workspace(const dfs_plan* P, int which, void** dev, int64_t* rows, int64_t* cols, int64_t* ld,
+                              int* dtype) {
+  if (!P || !dev || !rows || !cols || !ld || !dtype) return fail(DFS_EINVAL, "NULL argument");
+  const int s = P->last_step < 0 ? 0 : P->last_step, l = P->last_layer < 0 ? 0 : P->last_layer;
+  const StepLayer& S = P->sl[s * P->L + l];
+  const long long N = P->N, d = P->cfg.dim, hd = static_cast<long long>(S.h_s) * P->cfg.head_dim;
+  *dtype = 0;
+  switch (which) {
+    case 0: *dev = P->xm; *rows = N; *cols = d; *ld = d; break;
+    case 1: *dev = P->qk; *rows = N; *cols = 2 * hd; *ld = 2 * hd; break;
+    case 2: *dev = P->vt; *rows = hd; *cols = N; *ld = P->vt_ld; break;
+    case 3: *dev = P->attn; *rows = N; *cols = hd; *ld = hd; break;
+    case 4: *dev = P->x1; *rows = N; *cols = d; *ld = d; *dtype = 1; break;
+    case 5: *dev = P->h; *rows = N; *cols = S.f_s; *ld = S.f_s; break;
+    case 6: *dev = P->mod; *rows = 6; *cols = d; *ld = d; *dtype = 1; break;
+    default: return fail(DFS_EINVAL, "bad workspace id");
+  }
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_sync(dfs_plan* P, void* stream) {
+  if (!P) return fail(DFS_EINVAL, "plan is NULL");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  DFS_CK(cudaStreamSynchronize(st));
+  int herr = 0;
+  DFS_CK(cudaMemcpy(&herr, P->err, sizeof(int), cudaMemcpyDeviceToHost));
+  if (herr) {
+    DFS_CK(cudaMemset(P->err, 0, sizeof(int)));
+    return fail(DFS_ETIMEOUT, "a kernel gave up on a bounded wait (error word %d)", herr);
+  }
+  return DFS_OK;
+}
+
+dfs_status dfs_gates_from_soft_masks(int kind, int n_rows, int n_units, int unit_size, const float* m, uint8_t* g) {
+  if (!m || !g) return fail(DFS_EINVAL, "NULL m or g");
+  if (n_rows < 0 || n_units < 0 || unit_size < 1) return fail(DFS_EINVAL, "bad sizes");
+  if (kind != 1 && unit_size != 1) return fail(DFS_EINVAL, "unit_size must be 1 for block and FFN gates");
+  if (kind < 0 || kind > 2) return fail(DFS_EINVAL, "kind must be 0, 1 or 2");
+  for (long long r = 0; r < n_rows; ++r)
+    for (long long u = 0; u < n_units; ++u) {
+      const float* p = m + (r * n_units + u) * unit_size;
+      double sum = 0.0;
+      for (int i = 0; i < unit_size; ++i) sum += static_cast<double>(p[i]);
+      g[r * n_units + u] = (sum / unit_size > 0.0) ? 1 : 0;
+    }
+  return DFS_OK;
+}
+
+void dfs_plan_destroy(dfs_plan* plan) {
+  if (!plan) return;
+  cudaDeviceSynchronize();
+  free_plan(plan);
+}
+
+const char* dfs_last_error(void) { return g_last_error.c_str(); }
+
+}  // extern "C"

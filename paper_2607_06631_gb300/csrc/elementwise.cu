@@ -1,0 +1,370 @@
+// Memory-bound kernels of the block: weight compaction (K1), adaLN LayerNorm + modulate
+// and affine LayerNorm (K2 / K7), QK RMSNorm + 3D RoPE (K3), the modulation GEMV (K6),
+// bias-only residual branches and the Euler update (K8).  All move 16-byte vectors and
+// reduce with warp shuffles.
+#include "kernels.cuh"
+
+namespace dfs {
+namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Sum over the whole CTA (blockDim.x a multiple of 32, at most 1024); every thread gets it.
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  v = warp_sum(v);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = (l < nw) ? red[l] : 0.f;
+  return warp_sum(t);
+}
+
+// ------------------------------------------------------------------ K1 compaction
+
+__global__ void gather_rows_kernel(bf16* __restrict__ dst, long long ld_dst, const bf16* __restrict__ src,
+                                   long long ld_src, const int* __restrict__ rows, int n_rows, int vec_per_row) {
+  const long long total = static_cast<long long>(n_rows) * vec_per_row;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int r = static_cast<int>(i / vec_per_row);
+    const int v = static_cast<int>(i - static_cast<long long>(r) * vec_per_row);
+    const uint4 x = __ldg(reinterpret_cast<const uint4*>(src + rows[r] * ld_src) + v);
+    reinterpret_cast<uint4*>(dst + r * ld_dst)[v] = x;
+  }
+}
+
+__global__ void gather_segs_kernel(bf16* __restrict__ dst, long long ld_dst, const bf16* __restrict__ src,
+                                   long long ld_src, const int* __restrict__ seg, int n_seg, int n_rows) {
+  const long long total = static_cast<long long>(n_rows) * n_seg;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int r = static_cast<int>(i / n_seg);
+    const int j = static_cast<int>(i - static_cast<long long>(r) * n_seg);
+    const uint4 x = __ldg(reinterpret_cast<const uint4*>(src + r * ld_src) + seg[j]);
+    reinterpret_cast<uint4*>(dst + r * ld_dst)[j] = x;
+  }
+}
+
+int grid_for(long long work, int threads) {
+  long long g = (work + threads - 1) / threads;
+  if (g > 152LL * 16) g = 152LL * 16;
+  if (g < 1) g = 1;
+  return static_cast<int>(g);
+}
+
+// ------------------------------------------------------------------ K6 modulation GEMV
+
+__global__ void modulation_kernel(float* __restrict__ out, const bf16* __restrict__ W, const bf16* __restrict__ b,
+                                  const bf16* __restrict__ e, const bf16* __restrict__ t, int rows, int cols) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= rows) return;
+  const uint4* w4 = reinterpret_cast<const uint4*>(W + static_cast<long long>(warp) * cols);
+  const uint4* t4 = reinterpret_cast<const uint4*>(t);
+  float acc = 0.f;
+  for (int v = lane; v < cols / 8; v += 32) {
+    float a[8], x[8];
+    unpack_bf16x8(__ldg(w4 + v), a);
+    unpack_bf16x8(__ldg(t4 + v), x);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc = fmaf(a[i], x[i], acc);
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) {
+    float y = acc + bf16_to_f32(b[warp]);
+    if (e != nullptr) y += bf16_to_f32(e[warp]);
+    out[warp] = y;
+  }
+}
+
+__global__ void add_table_kernel(float* out, const float* base, const bf16* e, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) out[i] = base[i] + bf16_to_f32(e[i]);
+}
+
+// ------------------------------------------------------------------ K2 / K7 row LayerNorm
+
+constexpr int kNormThreads = 256;
+constexpr int kNormMaxVec = 4;  // up to 256 * 4 * 8 = 8192 columns
+
+template <bool F32IN>
+__global__ void __launch_bounds__(kNormThreads) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
+                                                                int cols, const float* __restrict__ mul,
+                                                                float mul_bias, const float* __restrict__ add,
+                                                                float eps) {
+  __shared__ float red[32];
+  const long long row = blockIdx.x;
+  const int nvec = cols >> 3;
+  float v[kNormMaxVec][8];
+  float s = 0.f;
+#pragma unroll
+  for (int k = 0; k < kNormMaxVec; ++k) {
+    const int c = threadIdx.x + k * blockDim.x;
+    if (c < nvec) {
+      if (F32IN) {
+        const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(xv) + row * cols) + 2 * c;
+        const float4 a = p[0], b = p[1];
+        v[k][0] = a.x; v[k][1] = a.y; v[k][2] = a.z; v[k][3] = a.w;
+        v[k][4] = b.x; v[k][5] = b.y; v[k][6] = b.z; v[k][7] = b.w;
+      } else {
+        unpack_bf16x8(reinterpret_cast<const uint4*>(static_cast<const bf16*>(xv) + row * cols)[c], v[k]);
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) s += v[k][i];
+    }
+  }
+  const float mean = block_sum(s, red) / cols;
+  float q = 0.f;
+#pragma unroll
+  for (int k = 0; k < kNormMaxVec; ++k) {
+    const int c = threadIdx.x + k * blockDim.x;
+    if (c < nvec) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float d = v[k][i] - mean;
+        q += d * d;
+      }
+    }
+  }
+  const float rstd = rsqrtf(block_sum(q, red) / cols + eps);
+#pragma unroll
+  for (int k = 0; k < kNormMaxVec; ++k) {
+    const int c = threadIdx.x + k * blockDim.x;
+    if (c < nvec) {
+      const float4* m4 = reinterpret_cast<const float4*>(mul) + 2 * c;
+      const float4* a4 = reinterpret_cast<const float4*>(add) + 2 * c;
+      const float4 m0 = __ldg(m4), m1 = __ldg(m4 + 1), a0 = __ldg(a4), a1 = __ldg(a4 + 1);
+      const float mm[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+      const float aa[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      float o[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) o[i] = fmaf((v[k][i] - mean) * rstd, mul_bias + mm[i], aa[i]);
+      reinterpret_cast<uint4*>(y + row * cols)[c] = pack_bf16x8(o);
+    }
+  }
+}
+
+// ------------------------------------------------------------------ K3 QK RMSNorm + RoPE
+
+constexpr int kQkThreads = 256;
+constexpr int kQkMaxVec = 8;  // up to 256 * 8 * 8 = 16384 channels per row (q and k)
+
+struct QkParams {
+  bf16* buf;
+  long long ld;
+  int nq, nk;
+  const bf16* gq;
+  const bf16* gk;
+  int head_dim, mode;
+  float eps;
+  int rope;
+  RopeTables t;
+};
+
+__global__ void __launch_bounds__(kQkThreads) qk_norm_rope_kernel(const QkParams p) {
+  __shared__ float red[32];
+  const long long row = blockIdx.x;
+  bf16* base = p.buf + row * p.ld;
+  const int nvq = p.nq >> 3, nv = (p.nq + p.nk) >> 3;
+  const int vph = p.head_dim >> 3;  // vectors per head (8 or 16); divides 32
+  float v[kQkMaxVec][8];
+  float sq = 0.f, sk = 0.f;
+  float hs[kQkMaxVec];
+#pragma unroll
+  for (int k = 0; k < kQkMaxVec; ++k) {
+    const int c = threadIdx.x + k * kQkThreads;
+    float ss = 0.f;
+    if (c < nv) {
+      unpack_bf16x8(reinterpret_cast<const uint4*>(base)[c], v[k]);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ss += v[k][i] * v[k][i];
+      if (c < nvq) sq += ss; else sk += ss;
+    }
+    hs[k] = ss;
+  }
+  float rq = 0.f, rk = 0.f;
+  if (p.mode == 0) {
+    const float tq = block_sum(sq, red);
+    const float tk = block_sum(sk, red);
+    rq = p.nq > 0 ? rsqrtf(tq / p.nq + p.eps) : 0.f;
+    rk = p.nk > 0 ? rsqrtf(tk / p.nk + p.eps) : 0.f;
+  } else {
+    // per head: the vph threads holding one head are consecutive lanes of one warp
+#pragma unroll
+    for (int k = 0; k < kQkMaxVec; ++k) {
+      float t = hs[k];
+      for (int o = vph >> 1; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+      hs[k] = rsqrtf(t / p.head_dim + p.eps);
+    }
+  }
+  int f = 0, yy = 0, xx = 0;
+  if (p.rope) {
+    const int hw = p.t.grid_h * p.t.grid_w;
+    f = static_cast<int>(row / hw);
+    const int rem = static_cast<int>(row - static_cast<long long>(f) * hw);
+    yy = rem / p.t.grid_w;
+    xx = rem - yy * p.t.grid_w;
+  }
+#pragma unroll
+  for (int k = 0; k < kQkMaxVec; ++k) {
+    const int c = threadIdx.x + k * kQkThreads;
+    if (c < nv) {
+      const bool is_q = c < nvq;
+      const int ch0 = (is_q ? c : c - nvq) * 8;  // channel within the q or k part
+      const float r = p.mode == 0 ? (is_q ? rq : rk) : hs[k];
+      float g[8];
+      unpack_bf16x8(reinterpret_cast<const uint4*>(is_q ? p.gq : p.gk)[ch0 >> 3], g);
+      float o[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) o[i] = v[k][i] * r * g[i];
+      if (p.rope) {
+        const int j0 = (ch0 % p.head_dim) >> 1;  // first rotation pair of this vector
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int j = j0 + i;
+          float cs, sn;
+          if (j < p.t.p_t) {
+            cs = p.t.cos_t[f * p.t.p_t + j];
+            sn = p.t.sin_t[f * p.t.p_t + j];
+          } else if (j < p.t.p_t + p.t.p_h) {
+            const int jj = j - p.t.p_t;
+            cs = p.t.cos_h[yy * p.t.p_h + jj];
+            sn = p.t.sin_h[yy * p.t.p_h + jj];
+          } else {
+            const int jj = j - p.t.p_t - p.t.p_h;
+            cs = p.t.cos_w[xx * p.t.p_w + jj];
+            sn = p.t.sin_w[xx * p.t.p_w + jj];
+          }
+          const float a = o[2 * i], b = o[2 * i + 1];
+          o[2 * i] = a * cs - b * sn;
+          o[2 * i + 1] = a * sn + b * cs;
+        }
+      }
+      reinterpret_cast<uint4*>(base)[c] = pack_bf16x8(o);
+    }
+  }
+}
+
+// ------------------------------------------------------------------ bias-only branches, Euler
+
+template <bool RF32, bool OF32>
+__global__ void bias_residual_kernel(void* out, const void* res, const float* gate, const bf16* bias, int rows,
+                                     int cols) {
+  const long long total = static_cast<long long>(rows) * cols;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int c = static_cast<int>(i % cols);
+    const float r = RF32 ? static_cast<const float*>(res)[i] : bf16_to_f32(static_cast<const bf16*>(res)[i]);
+    const float g = gate ? gate[c] : 1.f;
+    const float y = fmaf(g, bf16_to_f32(bias[c]), r);
+    if (OF32) static_cast<float*>(out)[i] = y;
+    else static_cast<bf16*>(out)[i] = __float2bfloat16_rn(y);
+  }
+}
+
+__global__ void to_f32_kernel(float* out, const bf16* in, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) out[i] = bf16_to_f32(in[i]);
+}
+
+__global__ void euler_kernel(bf16* x, const bf16* v, float dt, long long nvec) {
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < nvec;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    float a[8], b[8];
+    unpack_bf16x8(reinterpret_cast<const uint4*>(x)[i], a);
+    unpack_bf16x8(reinterpret_cast<const uint4*>(v)[i], b);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) a[k] = fmaf(dt, b[k], a[k]);
+    reinterpret_cast<uint4*>(x)[i] = pack_bf16x8(a);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_gather_rows(bf16* dst, long long ld_dst, const bf16* src, long long ld_src, const int* rows,
+                               int n_rows, int cols, cudaStream_t s) {
+  if (n_rows <= 0 || cols <= 0) return cudaSuccess;
+  const long long work = static_cast<long long>(n_rows) * (cols / 8);
+  gather_rows_kernel<<<grid_for(work, 256), 256, 0, s>>>(dst, ld_dst, src, ld_src, rows, n_rows, cols / 8);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_segs(bf16* dst, long long ld_dst, const bf16* src, long long ld_src, const int* seg,
+                               int n_seg, int n_rows, cudaStream_t s) {
+  if (n_rows <= 0 || n_seg <= 0) return cudaSuccess;
+  const long long work = static_cast<long long>(n_rows) * n_seg;
+  gather_segs_kernel<<<grid_for(work, 256), 256, 0, s>>>(dst, ld_dst, src, ld_src, seg, n_seg, n_rows);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_modulation(float* out, const bf16* W, const bf16* b, const bf16* e, const bf16* t, int rows,
+                              int cols, cudaStream_t s) {
+  const int threads = 256;
+  const int blocks = (rows * 32 + threads - 1) / threads;
+  modulation_kernel<<<blocks, threads, 0, s>>>(out, W, b, e, t, rows, cols);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_add_table(float* out, const float* base, const bf16* e, int n, cudaStream_t s) {
+  add_table_kernel<<<(n + 255) / 256, 256, 0, s>>>(out, base, e, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_row_norm(bf16* y, const void* x, int x_f32, int rows, int cols, const float* mul,
+                            float mul_bias, const float* add, float eps, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  if (cols % 8 != 0 || cols > kNormThreads * kNormMaxVec * 8) return cudaErrorInvalidValue;
+  int threads = ((cols / 8 + 31) / 32) * 32;
+  if (threads > kNormThreads) threads = kNormThreads;
+  if (x_f32)
+    row_norm_kernel<true><<<rows, threads, 0, s>>>(y, x, cols, mul, mul_bias, add, eps);
+  else
+    row_norm_kernel<false><<<rows, threads, 0, s>>>(y, x, cols, mul, mul_bias, add, eps);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_qk_norm_rope(bf16* buf, long long ld, int rows, int nq, int nk, const bf16* gamma_q,
+                                const bf16* gamma_k, int head_dim, int mode, float eps, const RopeTables* rope,
+                                cudaStream_t s) {
+  if (rows <= 0 || nq + nk <= 0) return cudaSuccess;
+  if ((nq + nk) / 8 > kQkThreads * kQkMaxVec || nq % head_dim || nk % head_dim) return cudaErrorInvalidValue;
+  QkParams p;
+  p.buf = buf; p.ld = ld; p.nq = nq; p.nk = nk; p.gq = gamma_q; p.gk = gamma_k;
+  p.head_dim = head_dim; p.mode = mode; p.eps = eps;
+  p.rope = rope != nullptr;
+  if (rope) p.t = *rope; else memset(&p.t, 0, sizeof(p.t));
+  qk_norm_rope_kernel<<<rows, kQkThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bias_residual(void* out, int out_f32, const void* res, int res_f32, const float* gate,
+                                 const bf16* bias, int rows, int cols, cudaStream_t s) {
+  const long long total = static_cast<long long>(rows) * cols;
+  if (total <= 0) return cudaSuccess;
+  const int g = grid_for(total, 256);
+  if (res_f32 && out_f32) bias_residual_kernel<true, true><<<g, 256, 0, s>>>(out, res, gate, bias, rows, cols);
+  else if (res_f32) bias_residual_kernel<true, false><<<g, 256, 0, s>>>(out, res, gate, bias, rows, cols);
+  else if (out_f32) bias_residual_kernel<false, true><<<g, 256, 0, s>>>(out, res, gate, bias, rows, cols);
+  else bias_residual_kernel<false, false><<<g, 256, 0, s>>>(out, res, gate, bias, rows, cols);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_to_f32(float* out, const bf16* in, int n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  to_f32_kernel<<<(n + 255) / 256, 256, 0, s>>>(out, in, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_euler(bf16* x, const bf16* v, float dt, long long n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const long long nvec = n / 8;
+  euler_kernel<<<grid_for(nvec, 256), 256, 0, s>>>(x, v, dt, nvec);
+  return cudaGetLastError();
+}
+
+}  // namespace dfs

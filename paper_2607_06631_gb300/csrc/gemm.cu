@@ -1,0 +1,298 @@
+// K4: persistent, warp-specialised tcgen05 GEMM for the block's projections
+// (QKV, attention output, FFN up / down), D = A * B^T with both operands K-major bf16.
+//
+//   warp 0      TMA producer: A tile 128x64 and B tile 256x64 per stage, 4-stage ring.
+//   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=256, K=16) into one of
+//               two TMEM accumulators (2 x 256 fp32 columns), so the epilogue of tile i
+//               overlaps the main loop of tile i+1.
+//   warps 2..5  epilogue: tcgen05.ld 32 columns at a time, fused bias / GELU / gated
+//               residual, predicated stores for the ragged M and N edges.
+// Ragged K (f_s is a multiple of 8, not of 64) is covered by TMA zero fill.
+#include "kernels.cuh"
+
+namespace dfs {
+namespace {
+
+__device__ __forceinline__ float gelu_tanh(float x) {
+  // GELU, tanh form: 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3)))
+  const float u = 0.7978845608028654f * fmaf(0.044715f * x, x * x, x);
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(u));
+  return 0.5f * x * (1.f + t);
+}
+
+// Grouped raster: 16 M-tiles share each sweep over N so that concurrent CTAs reuse
+// both operands from L2.
+__device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mt, int& nt) {
+  constexpr int G = 16;
+  const int group = tile / (G * n_tiles);
+  const int first_m = group * G;
+  const int gsz = min(m_tiles - first_m, G);
+  const int local = tile - group * G * n_tiles;
+  mt = first_m + local % gsz;
+  nt = local / gsz;
+}
+
+__device__ __forceinline__ void store_bf16_row(bf16* dst, const float (&v)[32], int valid) {
+  if (valid >= 32) {
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4 u;
+      u.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
+      u.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
+      u.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
+      u.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
+      d4[q] = u;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < valid) dst[j] = __float2bfloat16_rn(v[j]);
+  }
+}
+
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int row, int col0, float (&v)[32]) {
+  const int valid = min(32, p.N - col0);
+  if (p.bias != nullptr) {
+    if (valid >= 32) {
+      const uint4* b4 = reinterpret_cast<const uint4*>(p.bias + col0);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float f[8];
+        unpack_bf16x8(__ldg(b4 + q), f);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[8 * q + i] += f[i];
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < valid) v[j] += bf16_to_f32(p.bias[col0 + j]);
+    }
+  }
+  if (row >= p.M) return;
+
+  if (p.mode == kEpiBias) {
+    if (col0 < p.split) {
+      store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, valid);
+    } else {
+      bf16* t = p.out_t + static_cast<long long>(col0 - p.split) * p.ldt + row;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < valid) t[static_cast<long long>(j) * p.ldt] = __float2bfloat16_rn(v[j]);
+    }
+  } else if (p.mode == kEpiBiasGelu) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = gelu_tanh(v[j]);
+    store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, valid);
+  } else {  // kEpiGatedRes
+    float g[32], r[32];
+    if (p.gate != nullptr) {
+      if (valid >= 32) {
+        const float4* g4 = reinterpret_cast<const float4*>(p.gate + col0);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float4 t = __ldg(g4 + q);
+          g[4 * q] = t.x; g[4 * q + 1] = t.y; g[4 * q + 2] = t.z; g[4 * q + 3] = t.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) g[j] = (j < valid) ? p.gate[col0 + j] : 0.f;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) g[j] = 1.f;
+    }
+    if (p.res_f32) {
+      const float* rp = static_cast<const float*>(p.res) + static_cast<long long>(row) * p.ldr + col0;
+      if (valid >= 32) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float4 t = *reinterpret_cast<const float4*>(rp + 4 * q);
+          r[4 * q] = t.x; r[4 * q + 1] = t.y; r[4 * q + 2] = t.z; r[4 * q + 3] = t.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) r[j] = (j < valid) ? rp[j] : 0.f;
+      }
+    } else {
+      const bf16* rp = static_cast<const bf16*>(p.res) + static_cast<long long>(row) * p.ldr + col0;
+      if (valid >= 32) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          float f[8];
+          unpack_bf16x8(*reinterpret_cast<const uint4*>(rp + 8 * q), f);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) r[8 * q + i] = f[i];
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) r[j] = (j < valid) ? bf16_to_f32(rp[j]) : 0.f;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = fmaf(g[j], v[j], r[j]);
+    if (p.out_f32) {
+      float* op = static_cast<float*>(p.out) + static_cast<long long>(row) * p.ldo + col0;
+      if (valid >= 32) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          *reinterpret_cast<float4*>(op + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (j < valid) op[j] = v[j];
+      }
+    } else {
+      store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, valid);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __grid_constant__ GemmArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kGemmStages * kGemmABytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kGemmStages * kGemmStageBytes);
+  uint64_t* empty = full + kGemmStages;
+  uint64_t* tfull = empty + kGemmStages;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int m_tiles = (p.M + kGemmBM - 1) / kGemmBM;
+  const int n_tiles = (p.N + kGemmBN - 1) / kGemmBN;
+  const int num_tiles = m_tiles * n_tiles;
+  const int kb = (p.K + kGemmBK - 1) / kGemmBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kGemmStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 128);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  bool failed = false;
+
+  if (warp == 0) {
+    if (lane == 0 && kb > 0) {
+      tma_prefetch_desc(&p.tma_a);
+      tma_prefetch_desc(&p.tma_b);
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int tile = blockIdx.x; tile < num_tiles && !failed; tile += gridDim.x) {
+        int mt, nt;
+        tile_coords(tile, m_tiles, n_tiles, mt, nt);
+        for (int k = 0; k < kb; ++k) {
+          if (!mbar_wait(&empty[stage], phase ^ 1, p.err)) { failed = true; break; }
+          mbar_arrive_expect_tx(&full[stage], kGemmStageBytes);
+          tma_load_2d(sA + stage * kGemmABytes, &p.tma_a, &full[stage], k * kGemmBK, mt * kGemmBM);
+          tma_load_2d(sB + stage * kGemmBBytes, &p.tma_b, &full[stage], k * kGemmBK, nt * kGemmBN);
+          if (++stage == kGemmStages) { stage = 0; phase ^= 1; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && kb > 0) {
+      constexpr uint32_t idesc = idesc_bf16(kGemmBM, kGemmBN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int tile = blockIdx.x; tile < num_tiles && !failed; tile += gridDim.x) {
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, p.err)) { failed = true; break; }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * kGemmBN;
+        for (int k = 0; k < kb; ++k) {
+          if (!mbar_wait(&full[stage], phase, p.err)) { failed = true; break; }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * kGemmABytes);
+          const uint32_t b0 = smem_u32(sB + stage * kGemmBBytes);
+#pragma unroll
+          for (int kk = 0; kk < kGemmBK / 16; ++kk)
+            umma_bf16(d_tmem, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), idesc, (k | kk) != 0);
+          umma_commit(&empty[stage]);
+          if (++stage == kGemmStages) { stage = 0; phase ^= 1; }
+        }
+        umma_commit(&tfull[acc]);
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
+      }
+    }
+  } else {
+    const int sub = warp & 3;  // TMEM lane quarter this warp may access
+    const int r_in_tile = sub * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+      int mt, nt;
+      tile_coords(tile, m_tiles, n_tiles, mt, nt);
+      const int row = mt * kGemmBM + r_in_tile;
+      if (kb > 0) {
+        // every lane waits; the warp leaves together if any lane gave up, so that the
+        // warp-collective TMEM loads below are never split
+        const bool ok = mbar_wait(&tfull[acc], acc_phase, p.err);
+        if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+        tc_fence_after();
+      }
+      for (int c = 0; c < kGemmBN; c += 32) {
+        const int col0 = nt * kGemmBN + c;
+        if (col0 >= p.N) break;
+        float v[32];
+        if (kb > 0) {
+          tmem_ld32(tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * kGemmBN + c, v);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = 0.f;
+        }
+        epilogue_chunk(p, row, col0, v);
+      }
+      if (kb > 0) {
+        tc_fence_before();
+        mbar_arrive(&tempty[acc]);
+      }
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1;
+    }
+  }
+
+  if (failed) drain_after_error();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+}  // namespace
+
+cudaError_t gemm_prepare() {
+  return cudaFuncSetAttribute(gemm_bf16_tcgen05, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
+}
+
+cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t s) {
+  const int m_tiles = (a.M + kGemmBM - 1) / kGemmBM;
+  const int n_tiles = (a.N + kGemmBN - 1) / kGemmBN;
+  const int tiles = m_tiles * n_tiles;
+  if (tiles == 0) return cudaSuccess;
+  const int grid = tiles < num_sms ? tiles : num_sms;
+  gemm_bf16_tcgen05<<<grid, kGemmThreads, kGemmSmem, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace dfs

@@ -1,0 +1,107 @@
+// Argument structs and host launchers of every kernel of the library.  Launchers
+// enqueue on the given stream and return the launch's cudaError_t.
+#pragma once
+
+#include "common.cuh"
+
+namespace dfs {
+
+// ------------------------------------------------------------------------ K4 GEMM
+// D[M, N] = A[M, K] * B[N, K]^T with bf16 operands (both K-major), fp32 accumulation
+// in TMEM, and one of three fused epilogues.
+enum EpiMode : int {
+  kEpiBias = 0,      // out = acc + bias (bf16); columns >= split go transposed to out_t
+  kEpiBiasGelu = 1,  // out = GELU_tanh(acc + bias) (bf16)
+  kEpiGatedRes = 2,  // out = res + gate * (acc + bias) (res / out bf16 or fp32)
+};
+
+constexpr int kGemmBM = 128, kGemmBN = 256, kGemmBK = 64, kGemmStages = 4;
+constexpr int kGemmThreads = 192;
+constexpr int kGemmABytes = kGemmBM * kGemmBK * 2;
+constexpr int kGemmBBytes = kGemmBN * kGemmBK * 2;
+constexpr int kGemmStageBytes = kGemmABytes + kGemmBBytes;
+constexpr int kGemmSmem = kGemmStages * kGemmStageBytes + 1024 + 256;
+
+struct GemmArgs {
+  CUtensorMap tma_a;  // A [M, K], box {64, 128}, 128 B swizzle
+  CUtensorMap tma_b;  // B [N, K], box {64, 256}, 128 B swizzle
+  int M, N, K;
+  int mode;
+  const bf16* bias;  // [N] or null
+  void* out;
+  long long ldo;
+  int out_f32;
+  int split;         // kEpiBias: first column written transposed (multiple of 32); N = none
+  bf16* out_t;
+  long long ldt;
+  const void* res;   // kEpiGatedRes residual [M, ldr]
+  long long ldr;
+  int res_f32;
+  const float* gate;  // [N] or null (gate = 1)
+  int* err;
+};
+
+cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t s);
+cudaError_t gemm_prepare();  // opts the kernel into its shared-memory size
+
+// ------------------------------------------------------------------------ K5 attention
+// O[q, h*DH : (h+1)*DH] = softmax(Q_h K_h^T / sqrt(DH)) V_h for the retained heads.
+struct AttnArgs {
+  CUtensorMap tma_q;   // over the Q source, box {64, 128}
+  CUtensorMap tma_k;   // over the K source, box {64, 128}
+  CUtensorMap tma_vt;  // over V^T [heads*DH, n_kv], box {64, DH}
+  int n_q, n_kv, n_heads;
+  int q_col0, k_col0;  // column of head 0 in the Q / K sources
+  bf16* out;           // [n_q, ldo]
+  long long ldo;
+  float scale_log2;    // log2(e) / sqrt(DH)
+  int* err;
+};
+
+cudaError_t launch_attention(const AttnArgs& a, int head_dim, cudaStream_t s);
+cudaError_t attention_prepare();
+
+// ------------------------------------------------------------------------ memory-bound kernels
+
+// K1: dst[i, :] = src[rows[i], :] for i < n_rows (cols elements, multiple of 8).
+cudaError_t launch_gather_rows(bf16* dst, long long ld_dst, const bf16* src, long long ld_src,
+                               const int* rows, int n_rows, int cols, cudaStream_t s);
+// K1: dst[r, 8j : 8j+8] = src[r, 8*seg[j] : 8*seg[j]+8] for r < n_rows, j < n_seg.
+cudaError_t launch_gather_segs(bf16* dst, long long ld_dst, const bf16* src, long long ld_src,
+                               const int* seg, int n_seg, int n_rows, cudaStream_t s);
+
+// K6: out[r] = sum_c W[r, c] t[c] + b[r] (+ e[r]) for r < rows; W bf16 [rows, cols].
+cudaError_t launch_modulation(float* out, const bf16* W, const bf16* b, const bf16* e,
+                              const bf16* t, int rows, int cols, cudaStream_t s);
+// out[i] = base[i] + e[i] (e bf16), i < n.
+cudaError_t launch_add_table(float* out, const float* base, const bf16* e, int n, cudaStream_t s);
+
+// K2 / K7: y = (x - mean) * rstd * (mul_bias + mul[c]) + add[c], per row of `cols`;
+// x bf16 or fp32, y bf16.  mul / add fp32.
+cudaError_t launch_row_norm(bf16* y, const void* x, int x_f32, int rows, int cols, const float* mul,
+                            float mul_bias, const float* add, float eps, cudaStream_t s);
+
+// K3: in-place QK RMSNorm (+ 3D RoPE) on a row-major bf16 buffer: per row, channels
+// [0, nq) use gamma_q and [nq, nq + nk) use gamma_k; each part normalised on its own
+// (mode 0) or per head (mode 1); RoPE when rope_cos != null.
+struct RopeTables {
+  const float* cos_t; const float* sin_t;  // [G_t][p_t]
+  const float* cos_h; const float* sin_h;  // [G_h][p_h]
+  const float* cos_w; const float* sin_w;  // [G_w][p_w]
+  int grid_h, grid_w, p_t, p_h, p_w;
+};
+cudaError_t launch_qk_norm_rope(bf16* buf, long long ld, int rows, int nq, int nk, const bf16* gamma_q,
+                                const bf16* gamma_k, int head_dim, int mode, float eps,
+                                const RopeTables* rope, cudaStream_t s);
+
+// out[r, c] = res[r, c] + (gate ? gate[c] : 1) * bias[c]; res / out bf16 or fp32 (may alias).
+cudaError_t launch_bias_residual(void* out, int out_f32, const void* res, int res_f32, const float* gate,
+                                 const bf16* bias, int rows, int cols, cudaStream_t s);
+
+// out[i] = float(in[i]), i < n.
+cudaError_t launch_to_f32(float* out, const bf16* in, int n, cudaStream_t s);
+
+// K8: x = x + dt * v (bf16, n elements, n % 8 == 0).
+cudaError_t launch_euler(bf16* x, const bf16* v, float dt, long long n, cudaStream_t s);
+
+}  // namespace dfs

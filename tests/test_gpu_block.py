@@ -1,0 +1,158 @@
+"""GPU parity of the CUDA path (through the C ABI) against the float64 oracle."""
+import copy
+
+import numpy as np
+import pytest
+
+import oracle as O
+import synth
+from gpu_helpers import TOL, branch_err, check_block, rel_err, run_block
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2607_06631_gb300 import build
+    build.build()
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_tiny_every_step(mode):
+    cfg = synth.tiny(qk_norm_mode=mode)
+    r0, res = run_block(cfg)
+    check_block(cfg, r0, res)
+
+
+def test_tiny_index_lists_panels_and_flops_bit_exact():
+    from paper_2607_06631_gb300 import dfs, host
+    cfg = synth.tiny()
+    r0, _ = run_block(cfg, steps=[], want_intermediates=False)
+    plan, m, lw = r0["plan"], r0["masks"], r0["layers"][0]
+    for s in range(cfg.n_steps):
+        idx = O.compact_indices(cfg, m, s, 0)
+        np.testing.assert_array_equal(dfs.dfs_plan_indices(plan, s, 0, 0), idx["heads"])
+        np.testing.assert_array_equal(dfs.dfs_plan_indices(plan, s, 0, 1), idx["chunks"])
+        P = O.compact_panels(lw, idx)
+        for name in ("wqkv", "wo", "w_up", "w_down"):
+            np.testing.assert_array_equal(host.read_panel(plan, s, 0, name), P[name], err_msg=name)
+        for name in ("bqkv", "gq", "gk", "b_up"):
+            np.testing.assert_array_equal(host.read_panel(plan, s, 0, name)[0], P[name], err_msg=name)
+        f = O.block_flops(cfg.n_tokens, cfg.dim, cfg.head_dim, len(idx["heads"]), len(idx["ffn_ch"]))
+        assert dfs.dfs_plan_flops(plan, s, 0) == f
+
+
+def _custom(grid=(2, 16, 16), heads=(4, 3, 1, 2), chunks=(128, 9, 80, 64), dim=256, n_heads=4, ffn=1024,
+            head_dim=64):
+    cfg = synth.tiny(grid=grid)
+    cfg.dim, cfg.n_heads, cfg.head_dim, cfg.ffn_dim = dim, n_heads, head_dim, ffn
+    cfg.heads_kept = [[h] for h in heads]
+    cfg.chunks_kept = [[c] for c in chunks]
+    cfg.name = "custom_%s_%s_%s_%d" % ("x".join(map(str, grid)), "-".join(map(str, heads)),
+                                       "-".join(map(str, chunks)), head_dim)
+    return cfg
+
+
+@pytest.mark.parametrize("grid", [(1, 5, 7), (3, 10, 13), (1, 1, 8)])
+def test_ragged_token_counts(grid):
+    """N not a multiple of the 128-row tiles: 35, 390 and 8 tokens."""
+    cfg = _custom(grid=grid)
+    r0, res = run_block(cfg)
+    check_block(cfg, r0, res)
+
+
+def test_ragged_ffn_and_single_head():
+    """f_s = 72 (K tail of 8 inside a 64-wide K block), one retained head."""
+    cfg = _custom(heads=(1, 2, 1, 4), chunks=(9, 1, 33, 128))
+    r0, res = run_block(cfg)
+    check_block(cfg, r0, res)
+
+
+def test_head_dim_128_tiny():
+    cfg = _custom(dim=512, n_heads=4, head_dim=128, ffn=1024, heads=(4, 3, 2, 1), chunks=(128, 100, 50, 16),
+                  grid=(2, 8, 20))
+    r0, res = run_block(cfg)
+    check_block(cfg, r0, res)
+
+
+def test_empty_masks_and_block_gate():
+    cfg = synth.tiny()
+    m = synth.make_masks(cfg)
+    m["head_gate"][1, 0, :] = 0       # step 1: no heads -> x1 = x + gate_a * bo
+    m["ffn_gate"][2, 0, :] = 0        # step 2: no FFN chunks -> out = x1 + gate_f * b_down
+    m["head_gate"][3, 0, :] = 0
+    m["ffn_gate"][3, 0, :] = 0        # step 3: both empty
+    m["block_gate"][0, 0] = 0         # step 0: block off -> identity
+    r0, res = run_block(cfg, masks=m, want_intermediates=False)
+    check_block(cfg, r0, res, check_intermediates=False)
+    np.testing.assert_array_equal(res[0]["out"], r0["x"])
+
+
+def test_cross_attention_block():
+    cfg = synth.tiny(has_cross=1)
+    r0, res = run_block(cfg)
+    check_block(cfg, r0, res)
+
+
+def test_host_buffers_match_device_buffers():
+    import torch
+    from paper_2607_06631_gb300 import dfs, host
+    cfg = synth.tiny()
+    r0, _ = run_block(cfg, steps=[], want_intermediates=False)
+    plan, prob = r0["plan"], r0["prob"]
+    out = torch.empty_like(prob.x)
+    dfs.dfs_block_forward(plan, 2, prob.x, prob.t_emb[2], out)
+    dfs.dfs_plan_sync(plan)
+    x_h = prob.x.cpu().pin_memory()
+    t_h = prob.t_emb[2].cpu().pin_memory()
+    o_h = torch.empty_like(x_h).pin_memory()
+    dfs.dfs_block_forward_host(plan, 2, 0, x_h, t_h, o_h)
+    np.testing.assert_array_equal(host.to_bits(o_h), host.to_bits(out))
+
+
+def test_denoise_small_stack():
+    import torch
+    from paper_2607_06631_gb300 import dfs, host
+    cfg = synth.small_stack(4)
+    shared, layers, m, acts = synth.make_problem(cfg)
+    m["block_gate"][2, 1] = 0
+    prob = host.DeviceProblem(cfg, shared, layers, m, acts)
+    plan = prob.create_plan()
+    lat = prob.x.clone()
+    dfs.dfs_denoise(plan, lat, cfg.n_steps, prob.t_emb)
+    dfs.dfs_plan_sync(plan)
+    W, LW, X = synth.widen(shared), synth.widen(layers), synth.widen(acts)
+    ref = O.denoise(cfg, W, LW, m, X["x"], X["t_emb"], X["ctx"])
+    got = synth.bits_to_f64(host.to_bits(lat))
+    assert rel_err(got, ref) <= TOL
+    assert branch_err(got, ref, X["x"]) <= TOL
+
+
+def test_invalid_arguments_are_rejected():
+    import torch
+    from paper_2607_06631_gb300 import dfs
+    cfg = synth.tiny()
+    r0, _ = run_block(cfg, steps=[], want_intermediates=False)
+    plan, prob = r0["plan"], r0["prob"]
+    out = torch.empty_like(prob.x)
+    for args in ((4, 0), (-1, 0), (0, 1)):
+        with pytest.raises(dfs.DfsError) as e:
+            dfs.dfs_block_forward_layer(plan, args[0], args[1], prob.x, prob.t_emb[0], out)
+        assert e.value.status == dfs.DFS_EINVAL
+    with pytest.raises(dfs.DfsError) as e:
+        dfs.dfs_block_forward(plan, 0, prob.x, prob.t_emb[0], prob.x)
+    assert e.value.status == dfs.DFS_EINVAL
+
+
+def test_injected_allocation_failure(monkeypatch):
+    from paper_2607_06631_gb300 import dfs, host
+    cfg = synth.tiny()
+    shared, layers, m, acts = synth.make_problem(cfg)
+    prob = host.DeviceProblem(cfg, shared, layers, m, acts)
+    for n in (1, 7, 40):
+        monkeypatch.setenv("DFS_FAULT_ALLOC", str(n))
+        with pytest.raises(dfs.DfsError) as e:
+            prob.create_plan()
+        assert e.value.status == dfs.DFS_ENOMEM
+    monkeypatch.delenv("DFS_FAULT_ALLOC")
+    prob.create_plan()
