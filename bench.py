@@ -1,0 +1,405 @@
+#!/usr/bin/env python
+"""Benchmark of the step-specific pruned video-DiT block on GB300.
+
+One bench step = one pass of the whole hot path over one synthetic latent: the four
+distilled denoising steps of one Wan-14B-shaped block (d=5120, 40 heads x 128, FFN
+13824, 21x30x52 = 32760 tokens), each with its own retained heads / FFN chunks (keep
+1.0 / 0.8 / 0.7 / 0.55, i.e. 40/32/28/22 heads and 13824/11056/9680/7600 channels),
+run through the C ABI (dfs_block_forward).  Weights and inputs are seeded synthetic
+bf16 values (synth/), resident in HBM before timing; every input is larger than L2.
+
+Reported: TFLOP/s of algorithmic (pruned) FLOPs, its fraction of the measured bf16
+peak, the roofline of the dominant kernel (CUDA-event timed inside the timed region),
+the per-step pruned/dense speedup against the ideal FLOP ratio, an end-to-end number
+through the host-buffer entry point, and the CPU oracle's throughput on a bounded
+sample.  `--impl reference` times that CPU oracle alone (the reference arm).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "pruned-block TFLOP/s and % bf16 tensor peak; pruned/dense speedup vs ideal"
+KINDS = ("modulation", "adaln", "gemm_qkv", "qk_norm_rope", "attention", "gemm_o", "gemm_up", "gemm_down",
+         "cross", "other")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def get_config(name: str):
+    if name == "wan14b":
+        return synth.wan14b()
+    if name == "wan13b":
+        return synth.wan13b()
+    if name == "tiny":
+        return synth.tiny()
+    if name.startswith("sweep720:"):
+        return synth.sweep720(float(name.split(":")[1]))
+    raise SystemExit("unknown config " + name)
+
+
+def workload_desc(cfg) -> str:
+    hk = "/".join(str(cfg.heads_kept[s][0]) for s in range(cfg.n_steps))
+    fk = "/".join(str(8 * cfg.chunks_kept[s][0]) for s in range(cfg.n_steps))
+    return ("%s-shaped pruned DiT block, %d MoM steps per bench step: d=%d, %dx%d heads, FFN %d, "
+            "%s=%d tokens, kept heads %s, kept FFN channels %s"
+            % (cfg.name, cfg.n_steps, cfg.dim, cfg.n_heads, cfg.head_dim, cfg.ffn_dim,
+               "x".join(map(str, cfg.grid)), cfg.n_tokens, hk, fk))
+
+
+def kernel_units(cfg):
+    """Algorithmic work of each kernel kind summed over the MoM steps of one bench step:
+    ('tensor', FLOPs) or ('hbm', bytes)."""
+    N, d, dh = cfg.n_tokens, cfg.dim, cfg.head_dim
+    u = {k: 0.0 for k in KINDS}
+    for s in range(cfg.n_steps):
+        hd = cfg.heads_kept[s][0] * dh
+        fs = 8 * cfg.chunks_kept[s][0]
+        u["gemm_qkv"] += 2.0 * N * d * 3 * hd
+        u["attention"] += 4.0 * N * N * hd
+        u["gemm_o"] += 2.0 * N * hd * d
+        u["gemm_up"] += 2.0 * N * d * fs
+        u["gemm_down"] += 2.0 * N * fs * d
+        u["adaln"] += N * d * (2 + 2) + N * d * (4 + 2)      # x bf16 -> xm, x1 fp32 -> xm2
+        u["qk_norm_rope"] += 2.0 * N * 2 * hd * 2              # q, k read + written
+        u["modulation"] += 6.0 * d * d * 2                     # W_t read once
+    bound = {k: ("tensor" if k.startswith("gemm") or k == "attention" else "hbm") for k in KINDS}
+    return u, bound
+
+
+# ------------------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(gpu_index), "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.file, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [l.strip().split(",") for l in self.file.read().splitlines() if l.strip()]
+        self.file.close()
+        os.unlink(self.file.name)
+        sm, mx, reasons = [], 0.0, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx = max(mx, float(r[2]))
+                for n, v in zip(names, r[5:9]):
+                    if v.strip().lower().startswith("active"):
+                        reasons.add(n)
+            except (ValueError, IndexError):
+                continue
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx or None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------ distributed
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def dist_max(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ------------------------------------------------------------------------------ CPU oracle
+
+def cpu_cores() -> int:
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 0) for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def oracle_sample(cfg, problem_f64, step: int, rows: int, seed: int = 0):
+    """Runs the float64 oracle (compacted block) for `rows` query rows of one MoM step;
+    keys / values cover every token.  Returns (seconds, counted FLOPs)."""
+    import oracle as O
+    W, LW, M, X = problem_f64
+    r = np.sort(np.random.default_rng(seed).choice(cfg.n_tokens, size=rows, replace=False))
+    c = O.MacCounter()
+    t0 = time.perf_counter()
+    O.block_forward_compacted(cfg, W, LW[0], M, step, 0, X["x"], X["t_emb"][step], X.get("ctx"), rows=r,
+                              counter=c)
+    return time.perf_counter() - t0, c.flops
+
+
+def load_problem_f64(cfg):
+    shared, layers, masks, acts = synth.make_problem(cfg)
+    return synth.widen(shared), synth.widen(layers), masks, synth.widen(acts)
+
+
+CPU_ROWS = 32
+
+
+def cpu_baseline(cfg):
+    prob = load_problem_f64(cfg)
+    step = cfg.n_steps - 1
+    dt, fl = oracle_sample(cfg, prob, step, CPU_ROWS)
+    return {"value": fl / dt / 1e12, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
+            "sample": "float64 oracle, MoM step %d, %d query rows (keys/values over all %d tokens): "
+                      "%.3e counted FLOPs in %.1f s" % (step, CPU_ROWS, cfg.n_tokens, fl, dt)}
+
+
+def run_reference(args):
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return 0
+    cfg = get_config(args.config)
+    prob = load_problem_f64(cfg)
+    for i in range(args.warmup):
+        oracle_sample(cfg, prob, i % cfg.n_steps, CPU_ROWS, seed=1000 + i)
+    tot_t = tot_f = 0.0
+    for i in range(args.steps):
+        dt, fl = oracle_sample(cfg, prob, i % cfg.n_steps, CPU_ROWS, seed=i)
+        tot_t += dt
+        tot_f += fl
+    val = tot_f / tot_t / 1e12
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "TFLOP/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": workload_desc(cfg)},
+            "cpu_baseline": {"kind": "oracle", "cores": cpu_cores(), "value": val, "unit": "TFLOP/s",
+                             "sample": "each step: float64 oracle on one MoM step (cycling 0..3), %d query "
+                                       "rows, keys/values over all %d tokens" % (CPU_ROWS, cfg.n_tokens)},
+            "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------------------ our arm
+
+def run_ours(args):
+    import torch
+    world, rank, local = dist_setup()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    from paper_2607_06631_gb300 import build, dfs, host
+    build.build()
+    peaks, peak_src = load_peaks()
+    cfg = get_config(args.config)
+    T = cfg.n_steps
+    shared, layers, masks, acts = synth.make_problem(cfg)
+    prob = host.DeviceProblem(cfg, shared, layers, masks, acts)
+    del shared, layers
+    stream = torch.cuda.current_stream()
+    plan = prob.create_plan(stream)
+    prob.free_weights()
+    x, temb = prob.x, prob.t_emb
+    out = torch.empty_like(x)
+    flops = [dfs.dfs_plan_flops(plan, s) for s in range(T)]
+    flops_step = sum(flops)
+
+    def one_step():
+        for s in range(T):
+            dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
+
+    for _ in range(args.warmup):
+        one_step()
+    dfs.dfs_plan_sync(plan, stream)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    dfs.dfs_plan_profile(plan, True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        one_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    dfs.dfs_plan_profile(plan, False)
+    ck = clocks.stop()
+    barrier(world)
+    ms = e0.elapsed_time(e1)
+    ms_max = dist_max(ms, world)
+    value = flops_step * args.steps * world / (ms_max / 1e3) / 1e12
+    dfs.dfs_plan_sync(plan, stream)
+
+    # per-kernel event timings inside the timed region
+    units, bound = kernel_units(cfg)
+    kernels, launches = {}, 0
+    for k in KINDS:
+        kms, n = dfs.dfs_plan_profile_read(plan, k)
+        launches += n
+        if n == 0:
+            continue
+        work = units[k] * args.steps
+        if bound[k] == "tensor":
+            ach = work / (kms / 1e3) / 1e12
+            peak = peaks["bf16_tflops_sustained"]
+            unit = "TFLOP/s"
+        else:
+            ach = work / (kms / 1e3) / 1e9
+            peak = peaks["hbm_gbs"]
+            unit = "GB/s"
+        kernels[k] = {"launches": n, "ms_total": round(kms, 4), "ms_per_launch": round(kms / n, 5),
+                      "share": None, "achieved": round(ach, 2), "unit": unit, "peak": peak,
+                      "frac": round(ach / peak, 4), "bound": bound[k]}
+    tot_k = sum(v["ms_total"] for v in kernels.values())
+    for v in kernels.values():
+        v["share"] = round(v["ms_total"] / tot_k, 4)
+    dom = max(kernels, key=lambda k: kernels[k]["ms_total"])
+    dk = kernels[dom]
+    traffic = None
+    tfile = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tfile):
+        tr = json.load(open(tfile)).get(args.config, {}).get(dom)
+        if tr:
+            traffic = tr
+    roofline = {"kernel": dom, "bound": dk["bound"], "achieved": dk["achieved"], "peak": dk["peak"],
+                "unit": dk["unit"], "frac": dk["frac"], "traffic": traffic,
+                "peak_source": "%s (%s)" % (peak_src, "bf16_tflops_sustained" if dk["bound"] == "tensor"
+                                            else "hbm_gbs")}
+
+    # per-MoM-step latency: pruned vs dense (step 0 keeps every head and channel)
+    step_ms = []
+    reps = max(3, min(10, args.steps))
+    for s in range(T):
+        for _ in range(2):
+            dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        step_ms.append(a.elapsed_time(b) / reps)
+    speed = [step_ms[0] / t for t in step_ms]
+    ideal = [flops[0] / f for f in flops]
+    mean_meas = step_ms[0] / (sum(step_ms) / T)
+    mean_ideal = flops[0] / (sum(flops) / T)
+
+    # end to end through the host-buffer entry point (pinned host memory)
+    e2e = None
+    if not args.no_e2e:
+        xh = x.cpu().pin_memory()
+        th = temb.cpu().pin_memory()
+        oh = torch.empty_like(xh).pin_memory()
+        ke = max(1, min(args.steps, 5))
+        dfs.dfs_block_forward_host(plan, 0, 0, xh, th[0], oh, stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(ke):
+            for s in range(T):
+                dfs.dfs_block_forward_host(plan, s, 0, xh, th[s], oh, stream)
+        dt = time.perf_counter() - t0
+        dt = dist_max(dt, world)
+        nbytes = x.numel() * 2
+        e2e = {"value": flops_step * ke * world / dt / 1e12, "unit": "TFLOP/s",
+               "h2d_bytes_per_step": T * (nbytes + cfg.dim * 2), "d2h_bytes_per_step": T * nbytes,
+               "steps": ke}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        del prob
+        cpu = cpu_baseline(cfg)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": workload_desc(cfg), "l2": "inputs larger than L2 (x 335 MB, per-step "
+                       "weight panels 0.3-0.5 GB); no flush between steps",
+                       "parallelism": "replicas (one independent block per GPU)" if world > 1 else "1 GPU"},
+            "frac_of_peak": round(value / world / peaks["bf16_tflops_sustained"], 4),
+            "peak_tflops": peaks["bf16_tflops_sustained"], "peak_source": peak_src + " bf16_tflops_sustained",
+            "step_ms": [round(t, 4) for t in step_ms], "step_tflops": [round(f / t / 1e9, 1) for f, t in
+                                                                       zip(flops, step_ms)],
+            "speedup": [round(v, 4) for v in speed], "speedup_ideal": [round(v, 4) for v in ideal],
+            "speedup_vs_ideal": [round(a / b, 4) for a, b in zip(speed, ideal)],
+            "mean_speedup": round(mean_meas, 4), "mean_speedup_ideal": round(mean_ideal, 4),
+            "mean_speedup_vs_ideal": round(mean_meas / mean_ideal, 4),
+            "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": launches, "clocks": ck,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--config", default="wan14b", help="wan14b (default), wan13b, tiny, sweep720:<ratio>")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -147,6 +147,32 @@ dfs_status dfs_plan_workspace(const dfs_plan* plan, int which, void** dev, int64
  * Clears the plan's device error word. */
 dfs_status dfs_plan_sync(dfs_plan* plan, void* stream);
 
+/* Kernel kinds for dfs_plan_profile_read. */
+typedef enum {
+  DFS_K_MODULATION = 0,   /* adaLN modulation GEMV (W_t t_emb + b_t + E_l)          */
+  DFS_K_ADALN = 1,        /* LayerNorm + modulate (both norms of the block)           */
+  DFS_K_GEMM_QKV = 2,     /* QKV projection (bias epilogue, V written transposed)     */
+  DFS_K_QK_NORM_ROPE = 3, /* QK RMSNorm + 3D RoPE                                      */
+  DFS_K_ATTENTION = 4,    /* self-attention over the retained heads                    */
+  DFS_K_GEMM_O = 5,       /* output projection + gated residual                        */
+  DFS_K_GEMM_UP = 6,      /* FFN up projection + GELU                                  */
+  DFS_K_GEMM_DOWN = 7,    /* FFN down projection + gated residual                      */
+  DFS_K_CROSS = 8,        /* every kernel of the cross-attention branch                */
+  DFS_K_OTHER = 9,        /* bias-only branches, Euler update, block-gate copies       */
+  DFS_K_COUNT = 10
+} dfs_kernel_kind;
+
+/* Per-kernel timing of the forwards enqueued on this plan.  enable = 1 resets the
+ * counters and brackets every later kernel launch with a pair of CUDA events on its
+ * stream; enable = 0 stops recording (counters are kept).  Launch counts are kept in
+ * both modes.  Host only; no synchronisation. */
+dfs_status dfs_plan_profile(dfs_plan* plan, int enable);
+
+/* Sum of the event-measured durations (ms) and the launch count of one kernel kind
+ * since the last dfs_plan_profile(plan, 1).  Waits for the recorded events.
+ * total_ms is 0 for launches made while recording was off. */
+dfs_status dfs_plan_profile_read(dfs_plan* plan, int kind, double* total_ms, int64_t* launches);
+
 /* Soft mask -> hard gate rules of Sec. 4.1, host only (no CUDA call).
  * kind 0 = block: g = (m > 0); kind 1 = head: m holds unit_size entries per head and the
  * head is kept iff their mean (computed in double) is > 0; kind 2 = FFN chunk: one

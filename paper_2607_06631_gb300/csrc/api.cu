@@ -128,6 +128,12 @@ struct dfs_plan {
   std::vector<void*> allocs;
   int last_step = -1, last_layer = -1;
   int fault_alloc = -1, n_alloc = 0;  // host-side fault injection (DFS_FAULT_ALLOC=n)
+  // per-kernel profiling: event pairs recorded around launches while prof_on
+  bool prof_on = false;
+  std::vector<cudaEvent_t> ev;  // pool, pairs (2i, 2i+1)
+  std::vector<int> ev_kind;     // kind of each recorded pair
+  size_t ev_used = 0;
+  long long launches[DFS_K_COUNT] = {0};
 };
 
 namespace {
@@ -155,9 +161,45 @@ dfs_status alloc_n(dfs_plan* P, T** out, long long n) {
 
 void free_plan(dfs_plan* P) {
   if (!P) return;
+  for (cudaEvent_t e : P->ev) cudaEventDestroy(e);
   for (void* p : P->allocs) cudaFree(p);
   delete P;
 }
+
+// ------------------------------------------------------------------ per-kernel profiling
+
+// Brackets one kernel launch: records an event before and after it on `st` while
+// profiling is on, and counts the launch.
+struct ProfScope {
+  dfs_plan* P;
+  int kind;
+  cudaStream_t st;
+  int pair = -1;
+  ProfScope(dfs_plan* p, int k, cudaStream_t s) : P(p), kind(k), st(s) {
+    ++P->launches[kind];
+    if (!P->prof_on) return;
+    if (2 * P->ev_used + 2 > P->ev.size()) {
+      cudaEvent_t a, b;
+      if (cudaEventCreate(&a) != cudaSuccess) return;
+      if (cudaEventCreate(&b) != cudaSuccess) { cudaEventDestroy(a); return; }
+      P->ev.push_back(a);
+      P->ev.push_back(b);
+      P->ev_kind.push_back(kind);
+    }
+    pair = static_cast<int>(P->ev_used++);
+    P->ev_kind[pair] = kind;
+    cudaEventRecord(P->ev[2 * pair], st);
+  }
+  ~ProfScope() {
+    if (pair >= 0) cudaEventRecord(P->ev[2 * pair + 1], st);
+  }
+};
+
+#define DFS_LAUNCH(kind, expr)                \
+  do {                                        \
+    ProfScope prof_(P, (kind), st);           \
+    DFS_CK(expr);                             \
+  } while (0)
 
 // ------------------------------------------------------------------ validation (host only)
 
@@ -525,42 +567,42 @@ dfs_status forward_impl(dfs_plan* P, int s, int l, const bf16* x, bf16* out, cud
   P->last_step = s;
   P->last_layer = l;
 
-  DFS_CK(dfs::launch_row_norm(P->xm, x, 0, N, d, scale_a, 1.f, shift_a, c.ln_eps, st));
+  DFS_LAUNCH(DFS_K_ADALN, dfs::launch_row_norm(P->xm, x, 0, N, d, scale_a, 1.f, shift_a, c.ln_eps, st));
   if (S.h_s > 0) {
     const int hd = S.h_s * dh;
-    DFS_CK(dfs::launch_gemm(S.g_qkv, P->num_sms, st));
-    DFS_CK(dfs::launch_qk_norm_rope(P->qk, 2LL * hd, N, hd, hd, S.P[2].p, S.P[3].p, dh, c.qk_norm_mode, c.ln_eps,
+    DFS_LAUNCH(DFS_K_GEMM_QKV, dfs::launch_gemm(S.g_qkv, P->num_sms, st));
+    DFS_LAUNCH(DFS_K_QK_NORM_ROPE, dfs::launch_qk_norm_rope(P->qk, 2LL * hd, N, hd, hd, S.P[2].p, S.P[3].p, dh, c.qk_norm_mode, c.ln_eps,
                                     &P->rope, st));
-    DFS_CK(dfs::launch_attention(S.a_self, dh, st));
+    DFS_LAUNCH(DFS_K_ATTENTION, dfs::launch_attention(S.a_self, dh, st));
     dfs::GemmArgs g = S.g_o;
     g.res = x;
     g.gate = gate_a;
-    DFS_CK(dfs::launch_gemm(g, P->num_sms, st));
+    DFS_LAUNCH(DFS_K_GEMM_O, dfs::launch_gemm(g, P->num_sms, st));
   } else {
-    DFS_CK(dfs::launch_bias_residual(P->x1, 1, x, 0, gate_a, C.bo, N, d, st));
+    DFS_LAUNCH(DFS_K_OTHER, dfs::launch_bias_residual(P->x1, 1, x, 0, gate_a, C.bo, N, d, st));
   }
   if (c.has_cross) {
-    DFS_CK(dfs::launch_row_norm(P->xm, P->x1, 1, N, d, C.cln_w, 0.f, C.cln_b, c.ln_eps, st));
+    DFS_LAUNCH(DFS_K_CROSS, dfs::launch_row_norm(P->xm, P->x1, 1, N, d, C.cln_w, 0.f, C.cln_b, c.ln_eps, st));
     if (S.hc > 0) {
       const int hcd = S.hc * dh;
-      DFS_CK(dfs::launch_gemm(S.g_cq, P->num_sms, st));
-      DFS_CK(dfs::launch_qk_norm_rope(P->qc, hcd, N, hcd, 0, S.P[12].p, nullptr, dh, c.qk_norm_mode, c.ln_eps,
+      DFS_LAUNCH(DFS_K_CROSS, dfs::launch_gemm(S.g_cq, P->num_sms, st));
+      DFS_LAUNCH(DFS_K_CROSS, dfs::launch_qk_norm_rope(P->qc, hcd, N, hcd, 0, S.P[12].p, nullptr, dh, c.qk_norm_mode, c.ln_eps,
                                       nullptr, st));
-      DFS_CK(dfs::launch_attention(S.a_cross, dh, st));
-      DFS_CK(dfs::launch_gemm(S.g_co, P->num_sms, st));
+      DFS_LAUNCH(DFS_K_CROSS, dfs::launch_attention(S.a_cross, dh, st));
+      DFS_LAUNCH(DFS_K_CROSS, dfs::launch_gemm(S.g_co, P->num_sms, st));
     } else {
-      DFS_CK(dfs::launch_bias_residual(P->x1, 1, P->x1, 1, nullptr, C.cbo, N, d, st));
+      DFS_LAUNCH(DFS_K_CROSS, dfs::launch_bias_residual(P->x1, 1, P->x1, 1, nullptr, C.cbo, N, d, st));
     }
   }
-  DFS_CK(dfs::launch_row_norm(P->xm, P->x1, 1, N, d, scale_f, 1.f, shift_f, c.ln_eps, st));
+  DFS_LAUNCH(DFS_K_ADALN, dfs::launch_row_norm(P->xm, P->x1, 1, N, d, scale_f, 1.f, shift_f, c.ln_eps, st));
   if (S.f_s > 0) {
-    DFS_CK(dfs::launch_gemm(S.g_up, P->num_sms, st));
+    DFS_LAUNCH(DFS_K_GEMM_UP, dfs::launch_gemm(S.g_up, P->num_sms, st));
     dfs::GemmArgs g = S.g_down;
     g.out = out;
     g.gate = gate_f;
-    DFS_CK(dfs::launch_gemm(g, P->num_sms, st));
+    DFS_LAUNCH(DFS_K_GEMM_DOWN, dfs::launch_gemm(g, P->num_sms, st));
   } else {
-    DFS_CK(dfs::launch_bias_residual(out, 0, P->x1, 1, gate_f, C.bdown, N, d, st));
+    DFS_LAUNCH(DFS_K_OTHER, dfs::launch_bias_residual(out, 0, P->x1, 1, gate_f, C.bdown, N, d, st));
   }
   return DFS_OK;
 }
@@ -578,10 +620,10 @@ dfs_status block_layer(dfs_plan* P, int step, int layer, const bf16* x, const bf
                        cudaStream_t st) {
   const int d = P->cfg.dim;
   if (!P->block_gate[static_cast<size_t>(step) * P->L + layer]) {
-    DFS_CK(cudaMemcpyAsync(out, x, sizeof(bf16) * P->N * d, cudaMemcpyDeviceToDevice, st));
+    DFS_LAUNCH(DFS_K_OTHER, cudaMemcpyAsync(out, x, sizeof(bf16) * P->N * d, cudaMemcpyDeviceToDevice, st));
     return DFS_OK;
   }
-  DFS_CK(dfs::launch_modulation(P->mod, P->w_t, P->b_t, P->lc[layer].emod, t_emb, 6 * d, d, st));
+  DFS_LAUNCH(DFS_K_MODULATION, dfs::launch_modulation(P->mod, P->w_t, P->b_t, P->lc[layer].emod, t_emb, 6 * d, d, st));
   return forward_impl(P, step, layer, x, out, st);
 }
 
@@ -652,19 +694,20 @@ dfs_status dfs_denoise(dfs_plan* P, void* latents, int n_steps, const void* t_em
   const bf16* temb = static_cast<const bf16*>(t_embs);
   for (int s = 0; s < n_steps; ++s) {
     float* base = P->mod_base + 6LL * d * s;
-    DFS_CK(dfs::launch_modulation(base, P->w_t, P->b_t, nullptr, temb + static_cast<long long>(s) * d, 6 * d, d, st));
+    DFS_LAUNCH(DFS_K_MODULATION,
+               dfs::launch_modulation(base, P->w_t, P->b_t, nullptr, temb + static_cast<long long>(s) * d, 6 * d, d, st));
     const bf16* cur = lat;
     int ping = 0;
     for (int l = 0; l < P->L; ++l) {
       if (!P->block_gate[static_cast<size_t>(s) * P->L + l]) continue;
-      DFS_CK(dfs::launch_add_table(P->mod, base, P->lc[l].emod, 6 * d, st));
+      DFS_LAUNCH(DFS_K_MODULATION, dfs::launch_add_table(P->mod, base, P->lc[l].emod, 6 * d, st));
       bf16* dst = P->act[ping];
       dfs_status e = forward_impl(P, s, l, cur, dst, st);
       if (e) return e;
       cur = dst;
       ping ^= 1;
     }
-    DFS_CK(dfs::launch_euler(lat, cur, 1.f / P->cfg.n_steps, static_cast<long long>(P->N) * d, st));
+    DFS_LAUNCH(DFS_K_OTHER, dfs::launch_euler(lat, cur, 1.f / P->cfg.n_steps, static_cast<long long>(P->N) * d, st));
   }
   return DFS_OK;
 }
@@ -728,6 +771,32 @@ dfs_status dfs_plan_sync(dfs_plan* P, void* stream) {
     DFS_CK(cudaMemset(P->err, 0, sizeof(int)));
     return fail(DFS_ETIMEOUT, "a kernel gave up on a bounded wait (error word %d)", herr);
   }
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_profile(dfs_plan* P, int enable) {
+  if (!P) return fail(DFS_EINVAL, "plan is NULL");
+  if (enable) {
+    P->ev_used = 0;
+    for (long long& n : P->launches) n = 0;
+  }
+  P->prof_on = enable != 0;
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_profile_read(dfs_plan* P, int kind, double* total_ms, int64_t* launches) {
+  if (!P || !total_ms || !launches) return fail(DFS_EINVAL, "NULL argument");
+  if (kind < 0 || kind >= DFS_K_COUNT) return fail(DFS_EINVAL, "bad kernel kind");
+  double t = 0.0;
+  for (size_t i = 0; i < P->ev_used; ++i) {
+    if (P->ev_kind[i] != kind) continue;
+    DFS_CK(cudaEventSynchronize(P->ev[2 * i + 1]));
+    float ms = 0.f;
+    DFS_CK(cudaEventElapsedTime(&ms, P->ev[2 * i], P->ev[2 * i + 1]));
+    t += ms;
+  }
+  *total_ms = t;
+  *launches = P->launches[kind];
   return DFS_OK;
 }
 

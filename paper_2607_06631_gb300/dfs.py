@@ -22,7 +22,11 @@ _STATUS = {0: "DFS_OK", 1: "DFS_EINVAL", 2: "DFS_ENOMEM", 3: "DFS_ECUDA", 4: "DF
 
 EXPORTED = ("dfs_plan_create", "dfs_block_forward", "dfs_block_forward_layer", "dfs_block_forward_host",
             "dfs_denoise", "dfs_plan_indices", "dfs_plan_panel", "dfs_plan_flops", "dfs_plan_workspace",
-            "dfs_plan_sync", "dfs_gates_from_soft_masks", "dfs_plan_destroy", "dfs_last_error")
+            "dfs_plan_sync", "dfs_plan_profile", "dfs_plan_profile_read", "dfs_gates_from_soft_masks",
+            "dfs_plan_destroy", "dfs_last_error")
+
+KERNEL_KINDS = ("modulation", "adaln", "gemm_qkv", "qk_norm_rope", "attention", "gemm_o", "gemm_up",
+                "gemm_down", "cross", "other")
 
 PANELS = {"wqkv": 0, "bqkv": 1, "gq": 2, "gk": 3, "wo": 4, "w_up": 5, "b_up": 6, "w_down": 7,
           "cwq": 8, "cbq": 9, "cwkv": 10, "cbkv": 11, "cgq": 12, "cgk": 13, "cwo": 14}
@@ -76,6 +80,8 @@ def lib() -> ctypes.CDLL:
         L.dfs_plan_flops.argtypes = [vp, i32, i32, ctypes.POINTER(ctypes.c_double)]
         L.dfs_plan_workspace.argtypes = [vp, i32, ctypes.POINTER(vp), i64p, i64p, i64p, ctypes.POINTER(i32)]
         L.dfs_plan_sync.argtypes = [vp, vp]
+        L.dfs_plan_profile.argtypes = [vp, i32]
+        L.dfs_plan_profile_read.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_double), i64p]
         L.dfs_gates_from_soft_masks.argtypes = [i32, i32, i32, i32, vp, vp]
         L.dfs_plan_destroy.argtypes = [vp]
         L.dfs_plan_destroy.restype = None
@@ -238,6 +244,18 @@ def dfs_plan_workspace(plan, which):
 
 def dfs_plan_sync(plan, stream=None):
     _check(lib().dfs_plan_sync(_h(plan), _stream(stream)))
+
+
+def dfs_plan_profile(plan, enable: bool):
+    _check(lib().dfs_plan_profile(_h(plan), 1 if enable else 0))
+
+
+def dfs_plan_profile_read(plan, kind):
+    """(total event-timed ms, launches) of one kernel kind (index or name of KERNEL_KINDS)."""
+    k = KERNEL_KINDS.index(kind) if isinstance(kind, str) else kind
+    ms, n = ctypes.c_double(), ctypes.c_int64()
+    _check(lib().dfs_plan_profile_read(_h(plan), k, ctypes.byref(ms), ctypes.byref(n)))
+    return ms.value, n.value
 
 
 def dfs_gates_from_soft_masks(kind: int, m: np.ndarray, unit_size: int = 1) -> np.ndarray:

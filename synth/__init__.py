@@ -16,7 +16,9 @@ norm scales gamma = 1 + 0.1 N(0, 1); block input x, timestep embedding and text 
 """
 from __future__ import annotations
 
+import concurrent.futures as _cf
 import dataclasses
+import os
 import zlib
 from typing import Dict, List, Optional, Sequence
 
@@ -30,10 +32,11 @@ BASE_SEED = 20260706
 
 
 def f32_to_bf16_bits(a) -> np.ndarray:
-    """Round float32 values to bf16 (round to nearest, ties to even); returns uint16 bits."""
+    """Round finite float32 values to bf16 (round to nearest, ties to even); returns
+    uint16 bits.  (No finite float32 overflows the 32-bit sum below.)"""
     a = np.ascontiguousarray(np.asarray(a, dtype=np.float32))
-    u = a.view(np.uint32).astype(np.uint64)
-    u = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    u = a.view(np.uint32)
+    u = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)
     return u.astype(np.uint16)
 
 
@@ -154,14 +157,29 @@ def _rng(*parts) -> np.random.Generator:
     return np.random.Generator(np.random.PCG64(seed_for(*parts)))
 
 
+_CHUNK = 1 << 22
+_POOL = _cf.ThreadPoolExecutor(max_workers=max(1, min(32, os.cpu_count() or 1)))
+
+
 def normal_bits(shape, std=1.0, mean=0.0, *seed_parts) -> np.ndarray:
-    rng = _rng(*seed_parts)
-    a = rng.standard_normal(size=shape, dtype=np.float32)
-    if std != 1.0:
-        a *= np.float32(std)
-    if mean != 0.0:
-        a += np.float32(mean)
-    return f32_to_bf16_bits(a)
+    """bf16 bits of mean + std * N(0, 1) draws.  The tensor is filled in chunks of 2^22
+    values, chunk i from its own PCG64 stream seeded with (seed, i), in parallel threads."""
+    n = int(np.prod(shape)) if len(shape) else 1
+    out = np.empty(n, dtype=np.uint16)
+    base = seed_for(*seed_parts)
+
+    def fill(i):
+        lo, hi = i * _CHUNK, min(n, (i + 1) * _CHUNK)
+        rng = np.random.Generator(np.random.PCG64([base, i]))
+        a = rng.standard_normal(size=hi - lo, dtype=np.float32)
+        if std != 1.0:
+            a *= np.float32(std)
+        if mean != 0.0:
+            a += np.float32(mean)
+        out[lo:hi] = f32_to_bf16_bits(a)
+
+    list(_POOL.map(fill, range((n + _CHUNK - 1) // _CHUNK)))
+    return out.reshape(shape)
 
 
 LAYER_KEYS = ("wq", "bq", "wk", "bk", "wv", "bv", "wo", "bo", "gq", "gk",
