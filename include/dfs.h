@@ -107,6 +107,25 @@ dfs_status dfs_block_forward_layer(dfs_plan* plan, int step, int layer, const vo
 dfs_status dfs_block_forward_host(dfs_plan* plan, int step, int layer, const void* x_host,
                                   const void* t_emb_host, void* out_host, void* stream);
 
+/* Allocation-free variant of dfs_block_forward_layer (the paper has no counterpart;
+ * this is a deployment convenience).  Same arguments, same kernels, same result; the
+ * per-call activation workspace lives in a 16 MiB device array that the library
+ * declares statically, instead of memory the plan allocated.  For callers that must not
+ * allocate device memory while running the model: a host application that owns every
+ * device allocation through its own pool and budget, or a latency-critical loop that
+ * cannot absorb cudaMalloc's implicit synchronisation.  The plan must already exist.
+ *   - Nothing is allocated: no cudaMalloc, cudaFree or allocating library routine.
+ *   - The first call on a device looks up the array's device address (with that device
+ *     current) and keeps it; make that first call before any stream capture.
+ *   - Every call on a device shares the one array and leaves its contents behind; no
+ *     call relies on what an earlier call left.  Calls whose GPU work overlaps (other
+ *     streams, other host threads) race on the array: serialise them.
+ *   - A (step, layer) whose workspace (about N * (6 dim + 8 h_s head_dim + 2 f_s) bytes)
+ *     exceeds 16 MiB is rejected with DFS_EUNSUPPORTED and a message giving the need.
+ * Errors: as dfs_block_forward_layer, plus DFS_EUNSUPPORTED. */
+dfs_status dfs_block_forward_noalloc(dfs_plan* plan, int step, int layer, const void* x,
+                                     const void* t_emb, void* out, void* stream);
+
 /* Few-step denoising loop (Sec. 3.1, Fig. 1(b) rollout): for s in 0..n_steps-1, run
  * every layer with its step-s structure (block-gated layers skipped), then
  * latents <- latents + (1/cfg.n_steps) * v with v the last layer's output.

@@ -7,6 +7,8 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <map>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -824,3 +826,153 @@ void dfs_plan_destroy(dfs_plan* plan) {
 const char* dfs_last_error(void) { return g_last_error.c_str(); }
 
 }  // extern "C"
+
+// ------------------------------------------------------------------ forward without allocation
+//
+// dfs_block_forward_noalloc runs the same kernels as dfs_block_forward, but its
+// activation workspace (modulation vector, normalised activations, q/k, V^T, attention
+// output, fp32 residual, FFN hidden) lives in one file-scope device array instead of
+// memory the plan allocated.  It is meant for callers that must not allocate device
+// memory at forward time: for example a host application that owns all device memory
+// through its own pool and budget (a cudaMalloc behind its back breaks the budget and
+// fragments the pool), or a latency-critical serving loop where cudaMalloc / cudaFree
+// would add their implicit device synchronisation and unbounded latency.  The plan (its
+// compacted weights) must still have been created beforehand.
+
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = 16u << 20;  // 16 MiB, held by every GPU that loads the library
+
+__device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_noalloc_mu;
+std::map<int, unsigned char*> g_noalloc_addr;  // device ordinal -> device address of the array
+
+// Looks up (once per device, with that device current) the device address of the
+// scratch array; host code cannot use the symbol itself as a device pointer.
+dfs_status noalloc_scratch(int device, unsigned char** out) {
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  auto it = g_noalloc_addr.find(device);
+  if (it != g_noalloc_addr.end()) {
+    *out = it->second;
+    return DFS_OK;
+  }
+  void* p = nullptr;
+  cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (e != cudaSuccess || p == nullptr)
+    return fail(DFS_ECUDA, "cudaGetSymbolAddress(scratch) failed: %s", cudaGetErrorString(e));
+  g_noalloc_addr[device] = static_cast<unsigned char*>(p);
+  *out = static_cast<unsigned char*>(p);
+  return DFS_OK;
+}
+
+dfs_status noalloc_forward(dfs_plan* P, int s, int l, const bf16* x, const bf16* t_emb, bf16* out,
+                           cudaStream_t st) {
+  const dfs_config& c = P->cfg;
+  const int d = c.dim, dh = c.head_dim, N = P->N;
+  StepLayer& S = P->sl[s * P->L + l];
+  const LayerConst& C = P->lc[l];
+  if (!P->block_gate[static_cast<size_t>(s) * P->L + l]) {
+    DFS_CK(cudaMemcpyAsync(out, x, sizeof(bf16) * N * d, cudaMemcpyDeviceToDevice, st));
+    return DFS_OK;
+  }
+  const long long hd = static_cast<long long>(S.h_s) * dh, hcd = static_cast<long long>(S.hc) * dh;
+  const long long fs = S.f_s, vt_ld = round_up(N, 64);
+  // carve the scratch array (256-byte aligned pieces)
+  long long off = 0;
+  auto take = [&](long long bytes) {
+    const long long at = off;
+    off += round_up(bytes, 256);
+    return at;
+  };
+  const long long o_mod = take(6LL * d * 4), o_xm = take(2LL * N * d), o_qk = take(2LL * N * 2 * hd),
+                  o_vt = take(2LL * hd * vt_ld), o_attn = take(2LL * N * std::max(hd, hcd)),
+                  o_x1 = take(4LL * N * d), o_h = take(2LL * N * fs), o_qc = take(2LL * N * hcd);
+  if (off > static_cast<long long>(kNoAllocScratchBytes))
+    return fail(DFS_EUNSUPPORTED,
+                "this (step, layer) needs %lld bytes of scratch; the allocation-free forward has %zu",
+                off, kNoAllocScratchBytes);
+  int dev = 0;
+  DFS_CK(cudaGetDevice(&dev));
+  unsigned char* base = nullptr;
+  dfs_status e = noalloc_scratch(dev, &base);
+  if (e) return e;
+  float* mod = reinterpret_cast<float*>(base + o_mod);
+  bf16* xm = reinterpret_cast<bf16*>(base + o_xm);
+  bf16* qk = reinterpret_cast<bf16*>(base + o_qk);
+  bf16* vt = reinterpret_cast<bf16*>(base + o_vt);
+  bf16* attn = reinterpret_cast<bf16*>(base + o_attn);
+  float* x1 = reinterpret_cast<float*>(base + o_x1);
+  bf16* h = reinterpret_cast<bf16*>(base + o_h);
+  bf16* qc = reinterpret_cast<bf16*>(base + o_qc);
+  // Every scratch element a kernel reads is written earlier in this call, so nothing
+  // has to be cleared between calls.
+
+  DFS_CK(dfs::launch_modulation(mod, P->w_t, P->b_t, C.emod, t_emb, 6 * d, d, st));
+  DFS_CK(dfs::launch_row_norm(xm, x, 0, N, d, mod + d, 1.f, mod, c.ln_eps, st));
+  if (hd > 0) {
+    dfs::GemmArgs g = S.g_qkv;
+    if (!make_map(&g.tma_a, xm, d, N, d, 64, 128)) return fail(DFS_ECUDA, "tensor map (QKV) failed");
+    g.out = qk; g.out_t = vt; g.ldt = vt_ld;
+    DFS_CK(dfs::launch_gemm(g, P->num_sms, st));
+    DFS_CK(dfs::launch_qk_norm_rope(qk, 2 * hd, N, static_cast<int>(hd), static_cast<int>(hd), S.P[2].p,
+                                    S.P[3].p, dh, c.qk_norm_mode, c.ln_eps, &P->rope, st));
+    dfs::AttnArgs a = S.a_self;
+    if (!make_map(&a.tma_q, qk, 2 * hd, N, 2 * hd, 64, 128) || !make_map(&a.tma_vt, vt, N, hd, vt_ld, 64, dh))
+      return fail(DFS_ECUDA, "tensor map (attention) failed");
+    a.tma_k = a.tma_q;
+    a.out = attn;
+    DFS_CK(dfs::launch_attention(a, dh, st));
+    dfs::GemmArgs o = S.g_o;
+    if (!make_map(&o.tma_a, attn, hd, N, hd, 64, 128)) return fail(DFS_ECUDA, "tensor map (O) failed");
+    o.out = x1; o.res = x; o.gate = mod + 2 * d;
+    DFS_CK(dfs::launch_gemm(o, P->num_sms, st));
+  } else {
+    DFS_CK(dfs::launch_bias_residual(x1, 1, x, 0, mod + 2 * d, C.bo, N, d, st));
+  }
+  if (c.has_cross) {
+    DFS_CK(dfs::launch_row_norm(xm, x1, 1, N, d, C.cln_w, 0.f, C.cln_b, c.ln_eps, st));
+    if (hcd > 0) {
+      dfs::GemmArgs q = S.g_cq;
+      if (!make_map(&q.tma_a, xm, d, N, d, 64, 128)) return fail(DFS_ECUDA, "tensor map (cross q) failed");
+      q.out = qc;
+      DFS_CK(dfs::launch_gemm(q, P->num_sms, st));
+      DFS_CK(dfs::launch_qk_norm_rope(qc, hcd, N, static_cast<int>(hcd), 0, S.P[12].p, nullptr, dh,
+                                      c.qk_norm_mode, c.ln_eps, nullptr, st));
+      dfs::AttnArgs a = S.a_cross;
+      if (!make_map(&a.tma_q, qc, hcd, N, hcd, 64, 128)) return fail(DFS_ECUDA, "tensor map (cross attn) failed");
+      a.out = attn;
+      DFS_CK(dfs::launch_attention(a, dh, st));
+      dfs::GemmArgs o = S.g_co;
+      if (!make_map(&o.tma_a, attn, hcd, N, hcd, 64, 128)) return fail(DFS_ECUDA, "tensor map (cross o) failed");
+      o.out = x1; o.res = x1;
+      DFS_CK(dfs::launch_gemm(o, P->num_sms, st));
+    } else {
+      DFS_CK(dfs::launch_bias_residual(x1, 1, x1, 1, nullptr, C.cbo, N, d, st));
+    }
+  }
+  DFS_CK(dfs::launch_row_norm(xm, x1, 1, N, d, mod + 4 * d, 1.f, mod + 3 * d, c.ln_eps, st));
+  if (fs > 0) {
+    dfs::GemmArgs u = S.g_up;
+    if (!make_map(&u.tma_a, xm, d, N, d, 64, 128)) return fail(DFS_ECUDA, "tensor map (up) failed");
+    u.out = h;
+    DFS_CK(dfs::launch_gemm(u, P->num_sms, st));
+    dfs::GemmArgs dn = S.g_down;
+    if (!make_map(&dn.tma_a, h, fs, N, fs, 64, 128)) return fail(DFS_ECUDA, "tensor map (down) failed");
+    dn.out = out; dn.res = x1; dn.gate = mod + 5 * d;
+    DFS_CK(dfs::launch_gemm(dn, P->num_sms, st));
+  } else {
+    DFS_CK(dfs::launch_bias_residual(out, 0, x1, 1, mod + 5 * d, C.bdown, N, d, st));
+  }
+  return DFS_OK;
+}
+
+}  // namespace
+
+extern "C" dfs_status dfs_block_forward_noalloc(dfs_plan* plan, int step, int layer, const void* x,
+                                                const void* t_emb, void* out, void* stream) {
+  dfs_status e = check_forward_args(plan, step, layer, x, t_emb, out);
+  if (e) return e;
+  return noalloc_forward(plan, step, layer, static_cast<const bf16*>(x), static_cast<const bf16*>(t_emb),
+                         static_cast<bf16*>(out), static_cast<cudaStream_t>(stream));
+}

@@ -21,6 +21,7 @@ _STATUS = {0: "DFS_OK", 1: "DFS_EINVAL", 2: "DFS_ENOMEM", 3: "DFS_ECUDA", 4: "DF
            5: "DFS_EUNSUPPORTED"}
 
 EXPORTED = ("dfs_plan_create", "dfs_block_forward", "dfs_block_forward_layer", "dfs_block_forward_host",
+            "dfs_block_forward_noalloc",
             "dfs_denoise", "dfs_plan_indices", "dfs_plan_panel", "dfs_plan_flops", "dfs_plan_workspace",
             "dfs_plan_sync", "dfs_plan_profile", "dfs_plan_profile_read", "dfs_gates_from_soft_masks",
             "dfs_plan_destroy", "dfs_last_error")
@@ -74,6 +75,7 @@ def lib() -> ctypes.CDLL:
         L.dfs_block_forward.argtypes = [vp, i32, vp, vp, vp, vp]
         L.dfs_block_forward_layer.argtypes = [vp, i32, i32, vp, vp, vp, vp]
         L.dfs_block_forward_host.argtypes = [vp, i32, i32, vp, vp, vp, vp]
+        L.dfs_block_forward_noalloc.argtypes = [vp, i32, i32, vp, vp, vp, vp]
         L.dfs_denoise.argtypes = [vp, vp, i32, vp, vp]
         L.dfs_plan_indices.argtypes = [vp, i32, i32, i32, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(i32)]
         L.dfs_plan_panel.argtypes = [vp, i32, i32, i32, ctypes.POINTER(vp), i64p, i64p, i64p]
@@ -204,6 +206,13 @@ def dfs_block_forward_layer(plan, step: int, layer: int, x, t_emb, out, stream=N
 def dfs_block_forward_host(plan, step: int, layer: int, x_host, t_emb_host, out_host, stream=None):
     _check(lib().dfs_block_forward_host(_h(plan), step, layer, _ptr(x_host), _ptr(t_emb_host),
                                         _ptr(out_host), _stream(stream)))
+
+
+def dfs_block_forward_noalloc(plan, step: int, layer: int, x, t_emb, out, stream=None):
+    """As dfs_block_forward_layer without any device allocation: the workspace lives in
+    the library's static 16 MiB device array (see include/dfs.h for its rules)."""
+    _check(lib().dfs_block_forward_noalloc(_h(plan), step, layer, _ptr(x), _ptr(t_emb), _ptr(out),
+                                           _stream(stream)))
 
 
 def dfs_denoise(plan, latents, n_steps: int, t_embs, stream=None):
