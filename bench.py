@@ -46,7 +46,15 @@ def load_peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
-def get_config(name: str):
+def get_config(name: str, grid=None):
+    cfg = _named_config(name)
+    if grid:
+        cfg.grid = tuple(int(v) for v in grid.split(","))
+        cfg.name = cfg.name + "_grid" + "x".join(map(str, cfg.grid))
+    return cfg
+
+
+def _named_config(name: str):
     if name == "wan14b":
         return synth.wan14b()
     if name == "wan13b":
@@ -206,7 +214,7 @@ def run_reference(args):
     world, rank, _ = dist_setup()
     if rank != 0:
         return 0
-    cfg = get_config(args.config)
+    cfg = get_config(args.config, args.grid)
     prob = load_problem_f64(cfg)
     for i in range(args.warmup):
         oracle_sample(cfg, prob, i % cfg.n_steps, CPU_ROWS, seed=1000 + i)
@@ -242,7 +250,7 @@ def run_ours(args):
     from paper_2607_06631_gb300 import build, dfs, host
     build.build()
     peaks, peak_src = load_peaks()
-    cfg = get_config(args.config)
+    cfg = get_config(args.config, args.grid)
     T = cfg.n_steps
     shared, layers, masks, acts = synth.make_problem(cfg)
     prob = host.DeviceProblem(cfg, shared, layers, masks, acts)
@@ -393,6 +401,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--config", default="wan14b", help="wan14b (default), wan13b, tiny, sweep720:<ratio>")
+    ap.add_argument("--grid", default=None, help="override the latent grid T,H,W (smaller profiling cases)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()
