@@ -151,29 +151,29 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
     const int r = sub * 32 + lane;             // query row within the tile = TMEM lane
     const uint32_t lane_addr = static_cast<uint32_t>(sub * 32) << 16;
     const int q_row = q_tile * kBM + r;
-    float m_run = -INFINITY;                   // running max, log2 units
+    float m_run = -INFINITY;                   // running max of the scaled scores (log2 units)
     float l_run = 0.f;
+    const float sl2 = p.scale_log2;
     for (int j = 0; j < nkv; ++j) {
       const bool ok = mbar_wait(&s_full[j & 1], (j >> 1) & 1, p.err);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
       float s[kBN];
-#pragma unroll
-      for (int c = 0; c < kBN / 32; ++c) {
-        float t[32];
-        tmem_ld32(tmem + lane_addr + (j & 1) * kBN + c * 32, t);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) s[c * 32 + i] = t[i] * p.scale_log2;
-      }
+      tmem_ld128(tmem + lane_addr + (j & 1) * kBN, s);
       const int valid = p.n_kv - j * kBN;
       if (valid < kBN) {
 #pragma unroll
         for (int i = 0; i < kBN; ++i)
           if (i >= valid) s[i] = -INFINITY;
       }
-      float mx = s[0];
+      // row max with independent partial maxima (short dependency chains)
+      float pm[8];
 #pragma unroll
-      for (int i = 1; i < kBN; ++i) mx = fmaxf(mx, s[i]);
+      for (int i = 0; i < 8; ++i) pm[i] = s[i];
+#pragma unroll
+      for (int i = 8; i < kBN; ++i) pm[i & 7] = fmaxf(pm[i & 7], s[i]);
+      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * sl2;
 
       // PV_{j-1} must be complete before O is rescaled or P is overwritten.
       if (j > 0) {
@@ -188,30 +188,42 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
         const float alpha = move ? fast_exp2(m_run - mx) : 1.f;
         if (move) m_run = mx;
         l_run *= alpha;
+        // in halves of 64 columns; the scores are re-read from TMEM afterwards so that
+        // they need not stay live in registers across the rescale
 #pragma unroll
-        for (int c = 0; c < DH / 32; ++c) {
-          float o[32];
-          tmem_ld32(tmem_o + lane_addr + c * 32, o);
+        for (int c = 0; c < DH / 64; ++c) {
+          float o[64];
+          tmem_ld64(tmem_o + lane_addr + 64 * c, o);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tmem_st32(tmem_o + lane_addr + c * 32, o);
+          for (int i = 0; i < 64; ++i) o[i] *= alpha;
+          tmem_st64(tmem_o + lane_addr + 64 * c, o);
+        }
+        tmem_ld128(tmem + lane_addr + (j & 1) * kBN, s);
+        if (valid < kBN) {
+#pragma unroll
+          for (int i = 0; i < kBN; ++i)
+            if (i >= valid) s[i] = -INFINITY;
         }
       }
-      // P = exp2(s - m_run) -> bf16, 128-byte swizzled K-major layout for the P V MMA
-      float rs = 0.f;
+      // P = exp2(s * scale - m_run) -> bf16 in the 128-byte swizzled K-major layout of
+      // the P V operand; the row sum uses 8 independent partial sums.
+      const float neg_m = -m_run;
+      float ps[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ps[i] = 0.f;
 #pragma unroll
       for (int c = 0; c < kBN / 8; ++c) {
         float e[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          e[i] = fast_exp2(s[c * 8 + i] - m_run);
-          rs += e[i];
+          e[i] = fast_exp2(fmaf(s[c * 8 + i], sl2, neg_m));
+          ps[i] += e[i];
         }
         const int panel = c >> 3, chunk = c & 7;
         uint8_t* dst = sP + panel * (kBM * 128) + r * 128 + ((chunk ^ (r & 7)) << 4);
         *reinterpret_cast<uint4*>(dst) = pack_bf16x8(e);
       }
-      l_run += rs;
+      l_run += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
       fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(p_full);
@@ -223,19 +235,16 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
       } else {
         tc_fence_after();
         const float inv = 1.f / l_run;
-        bf16* dst = p.out + static_cast<long long>(q_row) * p.ldo + head * DH;
+        float o[DH];
+        if constexpr (DH == 128) tmem_ld128(tmem_o + lane_addr, o); else tmem_ld64(tmem_o + lane_addr, o);
+        if (q_row < p.n_q) {
+          bf16* dst = p.out + static_cast<long long>(q_row) * p.ldo + head * DH;
 #pragma unroll
-        for (int c = 0; c < DH / 32; ++c) {
-          float o[32];
-          tmem_ld32(tmem_o + lane_addr + c * 32, o);
-          if (q_row < p.n_q) {
+          for (int c = 0; c < DH / 8; ++c) {
+            float f[8];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              float f[8];
-#pragma unroll
-              for (int i = 0; i < 8; ++i) f[i] = o[8 * q + i] * inv;
-              *reinterpret_cast<uint4*>(dst + c * 32 + 8 * q) = pack_bf16x8(f);
-            }
+            for (int i = 0; i < 8; ++i) f[i] = o[8 * c + i] * inv;
+            *reinterpret_cast<uint4*>(dst + 8 * c) = pack_bf16x8(f);
           }
         }
       }
