@@ -57,6 +57,12 @@ def get_config(name: str, grid=None):
 def _named_config(name: str):
     if name == "wan14b":
         return synth.wan14b()
+    if name == "wan14b_cross":
+        return synth.wan14b_cross()
+    if name == "sweep720":
+        return synth.sweep720_all()
+    if name.startswith("wan14b_x"):
+        return synth.wan14b_stack(int(name[len("wan14b_x"):]))
     if name == "wan13b":
         return synth.wan13b()
     if name == "tiny":
@@ -69,10 +75,22 @@ def _named_config(name: str):
 def workload_desc(cfg) -> str:
     hk = "/".join(str(cfg.heads_kept[s][0]) for s in range(cfg.n_steps))
     fk = "/".join(str(8 * cfg.chunks_kept[s][0]) for s in range(cfg.n_steps))
-    return ("%s-shaped pruned DiT block, %d MoM steps per bench step: d=%d, %dx%d heads, FFN %d, "
-            "%s=%d tokens, kept heads %s, kept FFN channels %s"
-            % (cfg.name, cfg.n_steps, cfg.dim, cfg.n_heads, cfg.head_dim, cfg.ffn_dim,
-               "x".join(map(str, cfg.grid)), cfg.n_tokens, hk, fk))
+    what = ("%d-layer %d-step denoise (dfs_denoise)" % (cfg.n_layers, cfg.n_steps) if cfg.n_layers > 1
+            else "%d MoM steps per bench step" % cfg.n_steps)
+    cross = (", text cross-attention over %d context tokens (cross heads kept as self heads)" % cfg.ctx_len
+             if cfg.has_cross else "")
+    return ("%s-shaped pruned DiT block, %s: d=%d, %dx%d heads, FFN %d, %s=%d tokens, kept heads %s, "
+            "kept FFN channels %s%s"
+            % (cfg.name, what, cfg.dim, cfg.n_heads, cfg.head_dim, cfg.ffn_dim,
+               "x".join(map(str, cfg.grid)), cfg.n_tokens, hk, fk, cross))
+
+
+def panel_mb(cfg):
+    """Smallest and largest per-step compacted weight bytes of one layer (MB)."""
+    d, dh = cfg.dim, cfg.head_dim
+    mb = [(4 * cfg.heads_kept[s][0] * dh * d + 2 * 8 * cfg.chunks_kept[s][0] * d) * 2 / 1e6
+          for s in range(cfg.n_steps)]
+    return min(mb), max(mb)
 
 
 def kernel_units(cfg):
@@ -91,7 +109,13 @@ def kernel_units(cfg):
         u["adaln"] += N * d * (2 + 2) + N * d * (4 + 2)      # x bf16 -> xm, x1 fp32 -> xm2
         u["qk_norm_rope"] += 2.0 * N * 2 * hd * 2              # q, k read + written
         u["modulation"] += 6.0 * d * d * 2                     # W_t read once
-    bound = {k: ("tensor" if k.startswith("gemm") or k == "attention" else "hbm") for k in KINDS}
+        if cfg.has_cross:
+            hc = cfg.xheads_kept[s][0] * dh
+            u["cross"] += 4.0 * N * d * hc + 4.0 * N * cfg.ctx_len * hc
+    u = {k: v * cfg.n_layers for k, v in u.items()}
+    if cfg.n_layers > 1:  # the stack's modulation GEMV runs once per step, not per layer
+        u["modulation"] = cfg.n_steps * 6.0 * d * d * 2
+    bound = {k: ("tensor" if k.startswith("gemm") or k in ("attention", "cross") else "hbm") for k in KINDS}
     return u, bound
 
 
@@ -149,13 +173,21 @@ def dist_setup():
 
 
 def dist_max(x: float, world: int) -> float:
+    """Maximum of x over the ranks (timing only; the block itself exchanges nothing)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_value(flops_per_step: float, steps: int, world: int, ms_max: float) -> float:
+    """Whole-job TFLOP/s: every rank runs its own replica, so the units of all ranks are
+    divided by the slowest rank's time."""
+    return flops_per_step * steps * world / (ms_max / 1e3) / 1e12
 
 
 def barrier(world: int):
@@ -238,6 +270,34 @@ def run_reference(args):
 
 # ------------------------------------------------------------------------------ our arm
 
+def device_stack(cfg, seed: int = 20260706):
+    """Random-init weights of a multi-layer stack drawn directly on the device (torch
+    generator; N(0, 0.02) weights, 1 + 0.1 N(0, 1) norm scales): tens of GB would take
+    minutes through the host generator.  Masks, inputs and text context come from synth."""
+    import torch
+    from paper_2607_06631_gb300 import host
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+
+    def draw(shape, std, mean=0.0):
+        t = torch.empty(shape, device="cuda", dtype=torch.bfloat16)
+        t.normal_(mean, std, generator=g)
+        return t
+    layers = []
+    for _ in range(cfg.n_layers):
+        lw = {}
+        for k, shp in synth.layer_shapes(cfg).items():
+            scale = k in ("gq", "gk", "cgq", "cgk", "cln_w")
+            lw[k] = draw(shp, 0.1 if scale else 0.02, 1.0 if scale else 0.0)
+        layers.append(lw)
+    d = cfg.dim
+    w_t, b_t = draw((6 * d, d), 0.02), draw((6 * d,), 0.02)
+    acts = synth.make_activations(cfg)
+    x = host.to_device(acts["x"])
+    temb = host.to_device(acts["t_emb"])
+    ctx = host.to_device(acts["ctx"]) if "ctx" in acts else None
+    return layers, w_t, b_t, synth.make_masks(cfg), x, temb, ctx
+
 def run_ours(args):
     import torch
     world, rank, local = dist_setup()
@@ -251,21 +311,33 @@ def run_ours(args):
     build.build()
     peaks, peak_src = load_peaks()
     cfg = get_config(args.config, args.grid)
-    T = cfg.n_steps
-    shared, layers, masks, acts = synth.make_problem(cfg)
-    prob = host.DeviceProblem(cfg, shared, layers, masks, acts)
-    del shared, layers
+    T, L = cfg.n_steps, cfg.n_layers
     stream = torch.cuda.current_stream()
-    plan = prob.create_plan(stream)
-    prob.free_weights()
-    x, temb = prob.x, prob.t_emb
+    if L == 1:
+        shared, layers, masks, acts = synth.make_problem(cfg)
+        prob = host.DeviceProblem(cfg, shared, layers, masks, acts)
+        del shared, layers
+        plan = prob.create_plan(stream)
+        prob.free_weights()
+        x, temb = prob.x, prob.t_emb
+    else:
+        dl, w_t, b_t, masks, x, temb, ctx = device_stack(cfg)
+        plan = dfs.dfs_plan_create(cfg, dl, w_t, b_t, masks, ctx, stream)
+        del dl, w_t, b_t
+        torch.cuda.empty_cache()
+        prob = None
     out = torch.empty_like(x)
-    flops = [dfs.dfs_plan_flops(plan, s) for s in range(T)]
+    lat = x.clone()
+    flops = [sum(dfs.dfs_plan_flops(plan, s, l) for l in range(L)) for s in range(T)]
     flops_step = sum(flops)
 
     def one_step():
-        for s in range(T):
-            dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
+        if L == 1:
+            for s in range(T):
+                dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
+        else:
+            lat.copy_(x)
+            dfs.dfs_denoise(plan, lat, T, temb, stream)
 
     for _ in range(args.warmup):
         one_step()
@@ -285,7 +357,7 @@ def run_ours(args):
     barrier(world)
     ms = e0.elapsed_time(e1)
     ms_max = dist_max(ms, world)
-    value = flops_step * args.steps * world / (ms_max / 1e3) / 1e12
+    value = job_value(flops_step, args.steps, world, ms_max)
     dfs.dfs_plan_sync(plan, stream)
 
     # per-kernel event timings inside the timed region
@@ -326,8 +398,8 @@ def run_ours(args):
 
     # per-MoM-step latency: pruned vs dense (step 0 keeps every head and channel)
     step_ms = []
-    reps = max(3, min(10, args.steps))
-    for s in range(T):
+    reps = max(3, min(10, args.steps)) if L == 1 else 0
+    for s in (range(T) if L == 1 else ()):
         for _ in range(2):
             dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -337,14 +409,17 @@ def run_ours(args):
         b.record(stream)
         torch.cuda.synchronize()
         step_ms.append(a.elapsed_time(b) / reps)
-    speed = [step_ms[0] / t for t in step_ms]
     ideal = [flops[0] / f for f in flops]
-    mean_meas = step_ms[0] / (sum(step_ms) / T)
     mean_ideal = flops[0] / (sum(flops) / T)
+    if step_ms:
+        speed = [step_ms[0] / t for t in step_ms]
+        mean_meas = step_ms[0] / (sum(step_ms) / T)
+    else:  # the stack runs its steps inside dfs_denoise; per-step speedups are not separated
+        speed, mean_meas = None, None
 
     # end to end through the host-buffer entry point (pinned host memory)
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and L == 1:
         xh = x.cpu().pin_memory()
         th = temb.cpu().pin_memory()
         oh = torch.empty_like(xh).pin_memory()
@@ -364,7 +439,7 @@ def run_ours(args):
                "steps": ke}
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and L == 1:
         del prob
         cpu = cpu_baseline(cfg)
 
@@ -373,17 +448,21 @@ def run_ours(args):
             "metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": workload_desc(cfg), "l2": "inputs larger than L2 (x 335 MB, per-step "
-                       "weight panels 0.3-0.5 GB); no flush between steps",
+            "config": {"workload": workload_desc(cfg),
+                       "l2": "inputs larger than L2 (x %.0f MB, per-step weight panels %.0f-%.0f MB); no flush "
+                             "between steps" % (cfg.n_tokens * cfg.dim * 2 / 1e6, panel_mb(cfg)[0],
+                                                panel_mb(cfg)[1]),
                        "parallelism": "replicas (one independent block per GPU)" if world > 1 else "1 GPU"},
             "frac_of_peak": round(value / world / peaks["bf16_tflops_sustained"], 4),
             "peak_tflops": peaks["bf16_tflops_sustained"], "peak_source": peak_src + " bf16_tflops_sustained",
             "step_ms": [round(t, 4) for t in step_ms], "step_tflops": [round(f / t / 1e9, 1) for f, t in
                                                                        zip(flops, step_ms)],
-            "speedup": [round(v, 4) for v in speed], "speedup_ideal": [round(v, 4) for v in ideal],
-            "speedup_vs_ideal": [round(a / b, 4) for a, b in zip(speed, ideal)],
-            "mean_speedup": round(mean_meas, 4), "mean_speedup_ideal": round(mean_ideal, 4),
-            "mean_speedup_vs_ideal": round(mean_meas / mean_ideal, 4),
+            "speedup": [round(v, 4) for v in speed] if speed else None,
+            "speedup_ideal": [round(v, 4) for v in ideal],
+            "speedup_vs_ideal": [round(a / b, 4) for a, b in zip(speed, ideal)] if speed else None,
+            "mean_speedup": round(mean_meas, 4) if mean_meas else None,
+            "mean_speedup_ideal": round(mean_ideal, 4),
+            "mean_speedup_vs_ideal": round(mean_meas / mean_ideal, 4) if mean_meas else None,
             "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": ck,
         }
@@ -400,7 +479,9 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--config", default="wan14b", help="wan14b (default), wan13b, tiny, sweep720:<ratio>")
+    ap.add_argument("--config", default="wan14b",
+                    help="wan14b (default), wan13b, wan14b_cross, sweep720 (keep 1.0..0.5 as six steps), "
+                         "sweep720:<ratio>, wan14b_x<L> (L-layer 4-step denoise with cross-attention), tiny")
     ap.add_argument("--grid", default=None, help="override the latent grid T,H,W (smaller profiling cases)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")

@@ -136,6 +136,23 @@ def sweep720(ratio: float) -> Config:
                          (ratio,) * 4)
 
 
+SWEEP_RATIOS = (1.0, 0.9, 0.8, 0.7, 0.6, 0.5)
+
+
+def sweep720_all() -> Config:
+    """720p-shaped block whose six 'steps' are the uniform keep ratios 1.0 .. 0.5, so
+    one plan holds every point of the sweep (step i keeps SWEEP_RATIOS[i])."""
+    cfg = _ratio_config("sweep720", 5120, 40, 128, 13824, (21, 45, 80), SWEEP_RATIOS)
+    cfg.n_steps = len(SWEEP_RATIOS)
+    return cfg
+
+
+def wan14b_cross() -> Config:
+    """One Wan-14B-shaped block with text cross-attention over 512 context tokens."""
+    return _ratio_config("wan14b_cross", 5120, 40, 128, 13824, (21, 30, 52),
+                         (1.0, 0.8, 0.7, 0.55), has_cross=1, ctx_len=512)
+
+
 def small_stack(n_layers: int = 4) -> Config:
     """Shrunken stack (d=256, 2x8x8 tokens, cross-attention) for end-to-end denoise checks."""
     cfg = tiny(n_layers=n_layers, has_cross=1, grid=(2, 8, 8))

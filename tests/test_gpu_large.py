@@ -1,0 +1,74 @@
+"""GPU parity at the full benchmark sizes (Wan-1.3B- and Wan-14B-shaped blocks at 32760
+tokens, the 14B block with cross-attention, the 720p-shaped block at 75600 tokens).
+
+The CUDA path runs every token in the launch configuration bench.py times; the float64
+oracle computes the same block for a sample of query rows (keys / values still cover
+every token): the first and last rows (the last row tile is ragged: 32760 = 255*128+120,
+75600 = 590*128+80) and rows spread over the sequence."""
+import numpy as np
+import pytest
+
+import oracle as O
+import synth
+from gpu_helpers import TOL, branch_err, rel_err
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+
+def sample_rows(n, edge, spread, seed=0):
+    rng = np.random.default_rng(seed)
+    mid = rng.choice(np.arange(edge, n - edge), size=spread, replace=False)
+    return np.unique(np.concatenate([np.arange(edge), np.arange(n - edge, n), mid]))
+
+
+def run_large(cfg, steps, edge=64, spread=128):
+    import torch
+    from paper_2607_06631_gb300 import build, dfs, host
+    build.build()
+    shared, layers, masks, acts = synth.make_problem(cfg)
+    prob = host.DeviceProblem(cfg, shared, layers, masks, acts)
+    prob.create_plan()
+    prob.free_weights()
+    out = torch.empty_like(prob.x)
+    gpu = {}
+    for s in steps:
+        dfs.dfs_block_forward(prob.plan, s, prob.x, prob.t_emb[s], out)
+        dfs.dfs_plan_sync(prob.plan)
+        gpu[s] = out.clone()
+    del prob
+    torch.cuda.empty_cache()
+    W, LW, X = synth.widen(shared), synth.widen(layers), synth.widen(acts)
+    del shared, layers
+    rows = sample_rows(cfg.n_tokens, edge, spread)
+    errs = {}
+    for s in steps:
+        ref = O.block_forward_compacted(cfg, W, LW[0], masks, s, 0, X["x"], X["t_emb"][s], X.get("ctx"),
+                                        rows=rows)
+        got = synth.bits_to_f64(host.to_bits(gpu[s][torch.from_numpy(rows).cuda()]))
+        errs[s] = (rel_err(got, ref), branch_err(got, ref, X["x"][rows]))
+    return errs
+
+
+def test_wan13b_block_every_step():
+    errs = run_large(synth.wan13b(), range(4), edge=128, spread=256)
+    for s, (e, b) in errs.items():
+        assert e <= TOL and b <= TOL, (s, e, b)
+
+
+def test_wan14b_block_every_step():
+    errs = run_large(synth.wan14b(), range(4))
+    for s, (e, b) in errs.items():
+        assert e <= TOL and b <= TOL, (s, e, b)
+
+
+def test_wan14b_block_with_cross_attention():
+    errs = run_large(synth.wan14b_cross(), (0, 3), edge=32, spread=64)
+    for s, (e, b) in errs.items():
+        assert e <= TOL and b <= TOL, (s, e, b)
+
+
+def test_720p_block_half_keep():
+    cfg = synth.sweep720_all()
+    errs = run_large(cfg, (5,), edge=32, spread=64)  # step 5 keeps 20 heads / 6912 channels
+    for s, (e, b) in errs.items():
+        assert e <= TOL and b <= TOL, (s, e, b)
