@@ -166,6 +166,13 @@ dfs_status dfs_plan_workspace(const dfs_plan* plan, int which, void** dev, int64
  * Clears the plan's device error word. */
 dfs_status dfs_plan_sync(dfs_plan* plan, void* stream);
 
+/* Failure-path self test: launches one small kernel on `stream` that waits on a barrier
+ * nothing ever completes, through the same bounded wait every pipelined kernel of the
+ * library uses.  The wait gives up after about one second, records the timeout in the
+ * plan's device error word and returns, so the context stays usable; the next
+ * dfs_plan_sync reports DFS_ETIMEOUT (and clears the word).  No fault, trap or hang. */
+dfs_status dfs_selftest_wait_timeout(dfs_plan* plan, void* stream);
+
 /* Kernel kinds for dfs_plan_profile_read. */
 typedef enum {
   DFS_K_MODULATION = 0,   /* adaLN modulation GEMV (W_t t_emb + b_t + E_l)          */

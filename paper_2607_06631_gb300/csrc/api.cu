@@ -776,6 +776,12 @@ dfs_status dfs_plan_sync(dfs_plan* P, void* stream) {
   return DFS_OK;
 }
 
+dfs_status dfs_selftest_wait_timeout(dfs_plan* P, void* stream) {
+  if (!P) return fail(DFS_EINVAL, "plan is NULL");
+  DFS_CK(dfs::launch_wait_selftest(P->err, static_cast<cudaStream_t>(stream)));
+  return DFS_OK;
+}
+
 dfs_status dfs_plan_profile(dfs_plan* P, int enable) {
   if (!P) return fail(DFS_EINVAL, "plan is NULL");
   if (enable) {

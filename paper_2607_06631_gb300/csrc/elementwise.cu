@@ -272,6 +272,18 @@ __global__ void to_f32_kernel(float* out, const bf16* in, int n) {
   if (i < n) out[i] = bf16_to_f32(in[i]);
 }
 
+__global__ void wait_selftest_kernel(int* err) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  // nobody arrives on `bar`: the bounded wait runs out and records the timeout
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, err);
+  __syncthreads();
+}
+
 __global__ void euler_kernel(bf16* x, const bf16* v, float dt, long long nvec) {
   for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < nvec;
        i += static_cast<long long>(gridDim.x) * blockDim.x) {
@@ -357,6 +369,11 @@ cudaError_t launch_bias_residual(void* out, int out_f32, const void* res, int re
 cudaError_t launch_to_f32(float* out, const bf16* in, int n, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   to_f32_kernel<<<(n + 255) / 256, 256, 0, s>>>(out, in, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_selftest(int* err, cudaStream_t s) {
+  wait_selftest_kernel<<<1, 32, 0, s>>>(err);
   return cudaGetLastError();
 }
 

@@ -101,6 +101,9 @@ cudaError_t launch_bias_residual(void* out, int out_f32, const void* res, int re
 // out[i] = float(in[i]), i < n.
 cudaError_t launch_to_f32(float* out, const bf16* in, int n, cudaStream_t s);
 
+// Waits (bounded) on an mbarrier that nothing completes; sets *err to kErrTimeout.
+cudaError_t launch_wait_selftest(int* err, cudaStream_t s);
+
 // K8: x = x + dt * v (bf16, n elements, n % 8 == 0).
 cudaError_t launch_euler(bf16* x, const bf16* v, float dt, long long n, cudaStream_t s);
 

@@ -23,7 +23,7 @@ _STATUS = {0: "DFS_OK", 1: "DFS_EINVAL", 2: "DFS_ENOMEM", 3: "DFS_ECUDA", 4: "DF
 EXPORTED = ("dfs_plan_create", "dfs_block_forward", "dfs_block_forward_layer", "dfs_block_forward_host",
             "dfs_block_forward_noalloc",
             "dfs_denoise", "dfs_plan_indices", "dfs_plan_panel", "dfs_plan_flops", "dfs_plan_workspace",
-            "dfs_plan_sync", "dfs_plan_profile", "dfs_plan_profile_read", "dfs_gates_from_soft_masks",
+            "dfs_plan_sync", "dfs_selftest_wait_timeout", "dfs_plan_profile", "dfs_plan_profile_read", "dfs_gates_from_soft_masks",
             "dfs_plan_destroy", "dfs_last_error")
 
 KERNEL_KINDS = ("modulation", "adaln", "gemm_qkv", "qk_norm_rope", "attention", "gemm_o", "gemm_up",
@@ -82,6 +82,7 @@ def lib() -> ctypes.CDLL:
         L.dfs_plan_flops.argtypes = [vp, i32, i32, ctypes.POINTER(ctypes.c_double)]
         L.dfs_plan_workspace.argtypes = [vp, i32, ctypes.POINTER(vp), i64p, i64p, i64p, ctypes.POINTER(i32)]
         L.dfs_plan_sync.argtypes = [vp, vp]
+        L.dfs_selftest_wait_timeout.argtypes = [vp, vp]
         L.dfs_plan_profile.argtypes = [vp, i32]
         L.dfs_plan_profile_read.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_double), i64p]
         L.dfs_gates_from_soft_masks.argtypes = [i32, i32, i32, i32, vp, vp]
@@ -253,6 +254,10 @@ def dfs_plan_workspace(plan, which):
 
 def dfs_plan_sync(plan, stream=None):
     _check(lib().dfs_plan_sync(_h(plan), _stream(stream)))
+
+
+def dfs_selftest_wait_timeout(plan, stream=None):
+    _check(lib().dfs_selftest_wait_timeout(_h(plan), _stream(stream)))
 
 
 def dfs_plan_profile(plan, enable: bool):

@@ -156,3 +156,27 @@ def test_injected_allocation_failure(monkeypatch):
         assert e.value.status == dfs.DFS_ENOMEM
     monkeypatch.delenv("DFS_FAULT_ALLOC")
     prob.create_plan()
+
+
+def test_bounded_wait_reports_timeout_and_context_survives():
+    """A wait that nothing completes gives up after about a second, the host reads
+    DFS_ETIMEOUT, and the next forward on the same context is correct."""
+    import time
+    import torch
+    from paper_2607_06631_gb300 import dfs
+    cfg = synth.tiny()
+    r0, res = run_block(cfg, steps=[1], want_intermediates=False)
+    plan, prob = r0["plan"], r0["prob"]
+    t0 = time.time()
+    dfs.dfs_selftest_wait_timeout(plan)
+    with pytest.raises(dfs.DfsError) as e:
+        dfs.dfs_plan_sync(plan)
+    assert e.value.status == dfs.DFS_ETIMEOUT
+    assert time.time() - t0 < 30
+    dfs.dfs_plan_sync(plan)           # the error word was cleared
+    out = torch.empty_like(prob.x)
+    dfs.dfs_block_forward(plan, 1, prob.x, prob.t_emb[1], out)
+    dfs.dfs_plan_sync(plan)
+    from paper_2607_06631_gb300 import host
+    got = synth.bits_to_f64(host.to_bits(out))
+    assert rel_err(got, res[0]["ref"]) <= TOL
