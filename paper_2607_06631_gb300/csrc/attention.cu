@@ -1,38 +1,39 @@
 // K5: non-causal flash attention over the retained heads only, on tcgen05 tensor cores.
 //
-// One CTA = 128 query rows of one head.  Per key/value block j of 128 tokens:
-//   S_j = Q K_j^T      tcgen05.mma (M=128, N=128, K=DH) into TMEM (two S buffers)
-//   P_j = exp2(S_j * scale - m)   softmax warps, one query row per thread, bf16 into smem
-//   O  += P_j V_j      tcgen05.mma (M=128, N=DH, K=128) into a TMEM accumulator
-// V arrives pre-transposed (V^T [heads*DH, n_kv], written by the QKV projection's
-// epilogue) so both MMAs read K-major operands.  The running max is only moved when it
-// grows by more than 2^8 (exact: the same stale max enters O and the row sum); O is then
-// rescaled in TMEM before the next P V.  S_{j+1} is computed while the softmax of S_j
-// runs.
+// One CTA = two 128-row query tiles (Q0, Q1) of one head, sharing every key / value
+// tile.  Per key / value block j of 128 tokens and tile i:
+//   S_i = Q_i K_j^T      tcgen05.mma (M=128, N=128, K=DH), fp32 into TMEM
+//   P_i = exp2(S_i * scale - m_i)   softmax warpgroup i (thread = query row), bf16 written
+//                        back into the first 64 columns of S_i's TMEM region
+//   O_i += P_i V_j       tcgen05.mma with A read from TMEM (M=128, N=DH, K=128)
+// The single MMA thread issues  S0_j, PV1_{j-1}, S1_j, PV0_j, S0_{j+1}, PV1_j, ...  so the
+// softmax of one tile runs while the tensor core works on the other tile (a window of two
+// 128x128x128 MMAs).  V arrives pre-transposed (V^T [heads*DH, n_kv], written by the QKV
+// projection's epilogue) so every shared-memory operand is K-major.  The running max only
+// moves when it grows by more than 2^8 (exact: the same stale max enters O and the row
+// sum); O is then rescaled in TMEM.  K and V sit in separate two-deep rings.
 //
-//   warp 0      TMA: Q once, then K_j and V^T_j into a 2-stage ring
-//   warp 1      MMA issuer (single thread) + TMEM owner
-//   warps 2..5  softmax / rescale / output, thread = query row (TMEM lane)
+//   warp 0      TMA: Q0, Q1 once; K_j and V^T_j into their rings
+//   warp 1      MMA issuer (single thread) + TMEM owner (512 columns: S0, S1, O0, O1)
+//   warps 2..5  softmax / rescale / output of tile 0
+//   warps 6..9  softmax / rescale / output of tile 1
 #include "kernels.cuh"
 
 namespace dfs {
 namespace {
 
-constexpr int kBM = 128;   // query rows per CTA
+constexpr int kBM = 128;   // query rows per tile (two tiles per CTA)
 constexpr int kBN = 128;   // key / value rows per block
-constexpr int kStages = 2;
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
 constexpr float kRescaleThreshold = 8.f;  // log2 units
 
 template <int DH>
 struct AttnLayout {
-  static constexpr int kQBytes = kBM * DH * 2;
-  static constexpr int kKBytes = kBN * DH * 2;
-  static constexpr int kVBytes = DH * kBN * 2;
-  static constexpr int kPBytes = kBM * kBN * 2;
-  static constexpr int kStageBytes = kKBytes + kVBytes;
-  static constexpr int kSmem = kQBytes + kStages * kStageBytes + kPBytes + 1024 + 256;
-  static constexpr uint32_t kTmemCols = 512;  // S0 [0,128), S1 [128,256), O [256, 256+DH)
+  static constexpr int kQBytes = kBM * DH * 2;   // one query tile
+  static constexpr int kKBytes = kBN * DH * 2;   // one key tile
+  static constexpr int kVBytes = DH * kBN * 2;   // one V^T tile
+  static constexpr int kSmem = 2 * kQBytes + 2 * kKBytes + 2 * kVBytes + 1024 + 256;
+  static constexpr uint32_t kTmemCols = 512;     // S0 [0,128) S1 [128,256) O0 [256,..) O1 [384,..)
 };
 
 template <int DH>
@@ -40,34 +41,37 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
   using L = AttnLayout<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem;
-  uint8_t* sKV = sQ + L::kQBytes;  // stage s: K at s*kStageBytes, V^T after it
-  uint8_t* sP = sKV + kStages * L::kStageBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + L::kPBytes);
-  uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;              // [kStages]
-  uint64_t* kv_empty = kv_full + kStages;    // [kStages]
-  uint64_t* s_full = kv_empty + kStages;     // [2]
-  uint64_t* p_full = s_full + 2;
-  uint64_t* o_done = p_full + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_done + 1);
+  uint8_t* sQ = smem;                        // tile i at i * kQBytes
+  uint8_t* sK = sQ + 2 * L::kQBytes;         // ring slot b at b * kKBytes
+  uint8_t* sV = sK + 2 * L::kKBytes;         // ring slot b at b * kVBytes
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + 2 * L::kVBytes);
+  uint64_t* q_full = bars;                   // 1
+  uint64_t* k_full = bars + 1;               // [2]
+  uint64_t* k_empty = k_full + 2;            // [2]
+  uint64_t* v_full = k_empty + 2;            // [2]
+  uint64_t* v_empty = v_full + 2;            // [2]
+  uint64_t* s_full = v_empty + 2;            // [2] per tile: S_i of the current block ready
+  uint64_t* p_full = s_full + 2;             // [2] per tile: P_i written (and O_i rescaled)
+  uint64_t* o_done = p_full + 2;             // [2] per tile: last P_i V accumulated
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_done + 2);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int q_tile = blockIdx.x;
   const int head = blockIdx.y;
+  const int q_base = blockIdx.x * (2 * kBM);
   const int nkv = (p.n_kv + kBN - 1) / kBN;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&k_full[b], 1);
+      mbar_init(&k_empty[b], 1);
+      mbar_init(&v_full[b], 1);
+      mbar_init(&v_empty[b], 1);
+      mbar_init(&s_full[b], 1);
+      mbar_init(&p_full[b], 128);
+      mbar_init(&o_done[b], 1);
     }
-    mbar_init(&s_full[0], 1);
-    mbar_init(&s_full[1], 1);
-    mbar_init(p_full, 128);
-    mbar_init(o_done, 1);
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -78,7 +82,6 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tmem_o = tmem + 256;
   bool failed = false;
 
   if (warp == 0) {
@@ -88,22 +91,31 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
       tma_prefetch_desc(&p.tma_vt);
       const int qx = p.q_col0 + head * DH;
       const int kx = p.k_col0 + head * DH;
-      mbar_arrive_expect_tx(q_full, L::kQBytes);
+      mbar_arrive_expect_tx(q_full, 2 * L::kQBytes);
 #pragma unroll
-      for (int c = 0; c < DH / 64; ++c)
-        tma_load_2d(sQ + c * (kBM * 128), &p.tma_q, q_full, qx + 64 * c, q_tile * kBM);
-      for (int j = 0; j < nkv; ++j) {
-        const int s = j % kStages;
-        if (!mbar_wait(&kv_empty[s], ((j / kStages) & 1) ^ 1, p.err)) { failed = true; break; }
-        mbar_arrive_expect_tx(&kv_full[s], L::kStageBytes);
-        uint8_t* sK = sKV + s * L::kStageBytes;
-        uint8_t* sV = sK + L::kKBytes;
+      for (int i = 0; i < 2; ++i)
 #pragma unroll
         for (int c = 0; c < DH / 64; ++c)
-          tma_load_2d(sK + c * (kBN * 128), &p.tma_k, &kv_full[s], kx + 64 * c, j * kBN);
+          tma_load_2d(sQ + i * L::kQBytes + c * (kBM * 128), &p.tma_q, q_full, qx + 64 * c, q_base + i * kBM);
+      // K runs one block ahead of V: K_j is needed by S0_j long before V_j by PV0_j
+      for (int j = 0; j <= nkv && !failed; ++j) {
+        if (j < nkv) {
+          const int b = j & 1;
+          if (!mbar_wait(&k_empty[b], ((j >> 1) & 1) ^ 1, p.err)) { failed = true; break; }
+          mbar_arrive_expect_tx(&k_full[b], L::kKBytes);
 #pragma unroll
-        for (int c = 0; c < kBN / 64; ++c)
-          tma_load_2d(sV + c * (DH * 128), &p.tma_vt, &kv_full[s], j * kBN + 64 * c, head * DH);
+          for (int c = 0; c < DH / 64; ++c)
+            tma_load_2d(sK + b * L::kKBytes + c * (kBN * 128), &p.tma_k, &k_full[b], kx + 64 * c, j * kBN);
+        }
+        if (j >= 1) {
+          const int jv = j - 1, b = jv & 1;
+          if (!mbar_wait(&v_empty[b], ((jv >> 1) & 1) ^ 1, p.err)) { failed = true; break; }
+          mbar_arrive_expect_tx(&v_full[b], L::kVBytes);
+#pragma unroll
+          for (int c = 0; c < kBN / 64; ++c)
+            tma_load_2d(sV + b * L::kVBytes + c * (DH * 128), &p.tma_vt, &v_full[b], jv * kBN + 64 * c,
+                        head * DH);
+        }
       }
     }
   } else if (warp == 1) {
@@ -111,62 +123,85 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
       constexpr uint32_t idesc_s = idesc_bf16(kBM, kBN);
       constexpr uint32_t idesc_o = idesc_bf16(kBM, DH);
       const uint32_t q0 = smem_u32(sQ);
-      const uint32_t p0 = smem_u32(sP);
-      // S_j = Q K_j^T into S buffer (j & 1)
-      auto issue_s = [&](int j) -> bool {
-        const int s = j % kStages;
-        if (!mbar_wait(&kv_full[s], (j / kStages) & 1, p.err)) return false;
-        tc_fence_after();
-        const uint32_t k0 = smem_u32(sKV + s * L::kStageBytes);
+      // S_i(j) = Q_i K_j^T into S_i's TMEM columns
+      auto issue_s = [&](int i, int j) {
+        const uint32_t k0 = smem_u32(sK + (j & 1) * L::kKBytes);
+        const uint32_t qi = q0 + i * L::kQBytes;
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
           const uint32_t off = (kk / 4) * (kBM * 128) + (kk % 4) * 32;
-          const uint32_t offk = (kk / 4) * (kBN * 128) + (kk % 4) * 32;
-          umma_bf16(tmem + (j & 1) * kBN, sw128_desc(q0 + off), sw128_desc(k0 + offk), idesc_s, kk != 0);
+          umma_bf16(tmem + i * kBN, sw128_desc(qi + off), sw128_desc(k0 + off), idesc_s, kk != 0);
         }
-        umma_commit(&s_full[j & 1]);
-        return true;
+        umma_commit(&s_full[i]);
       };
-      if (!mbar_wait(q_full, 0, p.err)) failed = true;
-      if (!failed) failed = !issue_s(0);
-      if (!failed && nkv > 1) failed = !issue_s(1);
-      for (int j = 0; j < nkv && !failed; ++j) {
-        if (!mbar_wait(p_full, j & 1, p.err)) { failed = true; break; }
-        tc_fence_after();
-        const int s = j % kStages;
-        const uint32_t v0 = smem_u32(sKV + s * L::kStageBytes + L::kKBytes);
+      // O_i += P_i(j) V_j with P_i read from the first 64 columns of S_i
+      auto issue_pv = [&](int i, int j) {
+        const uint32_t v0 = smem_u32(sV + (j & 1) * L::kVBytes);
 #pragma unroll
         for (int kk = 0; kk < kBN / 16; ++kk) {
-          const uint32_t offp = (kk / 4) * (kBM * 128) + (kk % 4) * 32;
           const uint32_t offv = (kk / 4) * (DH * 128) + (kk % 4) * 32;
-          umma_bf16(tmem_o, sw128_desc(p0 + offp), sw128_desc(v0 + offv), idesc_o, (j | kk) != 0);
+          umma_bf16_tmem_a(tmem + 256 + i * 128, tmem + i * kBN + kk * 8, sw128_desc(v0 + offv), idesc_o,
+                           (j | kk) != 0);
         }
-        umma_commit(&kv_empty[s]);
-        umma_commit(o_done);
-        if (j + 2 < nkv) failed = !issue_s(j + 2);
-      }
+      };
+      do {
+        if (!mbar_wait(q_full, 0, p.err)) { failed = true; break; }
+        if (!mbar_wait(&k_full[0], 0, p.err)) { failed = true; break; }
+        tc_fence_after();
+        issue_s(0, 0);
+        issue_s(1, 0);
+        umma_commit(&k_empty[0]);
+        for (int j = 0; j < nkv; ++j) {
+          const int b = j & 1;
+          const uint32_t ph = (j >> 1) & 1;
+          // PV0_j
+          if (!mbar_wait(&p_full[0], j & 1, p.err) || !mbar_wait(&v_full[b], ph, p.err)) { failed = true; break; }
+          tc_fence_after();
+          issue_pv(0, j);
+          if (j + 1 == nkv) umma_commit(&o_done[0]);
+          // S0_{j+1}
+          if (j + 1 < nkv) {
+            if (!mbar_wait(&k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, p.err)) { failed = true; break; }
+            tc_fence_after();
+            issue_s(0, j + 1);
+          }
+          // PV1_j
+          if (!mbar_wait(&p_full[1], j & 1, p.err)) { failed = true; break; }
+          tc_fence_after();
+          issue_pv(1, j);
+          umma_commit(&v_empty[b]);
+          if (j + 1 == nkv) umma_commit(&o_done[1]);
+          // S1_{j+1}
+          if (j + 1 < nkv) {
+            issue_s(1, j + 1);
+            umma_commit(&k_empty[(j + 1) & 1]);
+          }
+        }
+      } while (false);
     }
   } else {
-    const int sub = warp & 3;
-    const int r = sub * 32 + lane;             // query row within the tile = TMEM lane
+    const int tile = (warp - 2) >> 2;        // 0: warps 2..5, 1: warps 6..9
+    const int sub = warp & 3;                // TMEM lane quarter this warp may access
+    const int r = sub * 32 + lane;           // query row within the tile = TMEM lane
     const uint32_t lane_addr = static_cast<uint32_t>(sub * 32) << 16;
-    const int q_row = q_tile * kBM + r;
-    float m_run = -INFINITY;                   // running max of the scaled scores (log2 units)
-    float l_run = 0.f;
+    const uint32_t tS = tmem + tile * kBN + lane_addr;
+    const uint32_t tO = tmem + 256 + tile * 128 + lane_addr;
+    const int q_row = q_base + tile * kBM + r;
     const float sl2 = p.scale_log2;
+    float m_run = -INFINITY;                 // running max of the scaled scores (log2 units)
+    float l_run = 0.f;
     for (int j = 0; j < nkv; ++j) {
-      const bool ok = mbar_wait(&s_full[j & 1], (j >> 1) & 1, p.err);
+      const bool ok = mbar_wait(&s_full[tile], j & 1, p.err);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
       float s[kBN];
-      tmem_ld128(tmem + lane_addr + (j & 1) * kBN, s);
+      tmem_ld128(tS, s);
       const int valid = p.n_kv - j * kBN;
       if (valid < kBN) {
 #pragma unroll
         for (int i = 0; i < kBN; ++i)
           if (i >= valid) s[i] = -INFINITY;
       }
-      // row max with independent partial maxima (short dependency chains)
       float pm[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) pm[i] = s[i];
@@ -174,77 +209,65 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
       for (int i = 8; i < kBN; ++i) pm[i & 7] = fmaxf(pm[i & 7], s[i]);
       const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
                              fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * sl2;
-
-      // PV_{j-1} must be complete before O is rescaled or P is overwritten.
-      if (j > 0) {
-        const bool ok2 = mbar_wait(o_done, (j - 1) & 1, p.err);
-        if (!__all_sync(0xffffffffu, ok2)) { failed = true; break; }
-        tc_fence_after();
-      }
       const bool move = mx > m_run + kRescaleThreshold;
       if (j == 0) {
         m_run = mx;
       } else if (__any_sync(0xffffffffu, move)) {
+        // S_i(j) completing implies P_i(j-1) V_{j-1} completed: O_i is stable here
         const float alpha = move ? fast_exp2(m_run - mx) : 1.f;
         if (move) m_run = mx;
         l_run *= alpha;
-        // in halves of 64 columns; the scores are re-read from TMEM afterwards so that
-        // they need not stay live in registers across the rescale
 #pragma unroll
-        for (int c = 0; c < DH / 64; ++c) {
-          float o[64];
-          tmem_ld64(tmem_o + lane_addr + 64 * c, o);
+        for (int c = 0; c < DH / 32; ++c) {
+          float o[32];
+          tmem_ld32(tO + 32 * c, o);
 #pragma unroll
-          for (int i = 0; i < 64; ++i) o[i] *= alpha;
-          tmem_st64(tmem_o + lane_addr + 64 * c, o);
-        }
-        tmem_ld128(tmem + lane_addr + (j & 1) * kBN, s);
-        if (valid < kBN) {
-#pragma unroll
-          for (int i = 0; i < kBN; ++i)
-            if (i >= valid) s[i] = -INFINITY;
+          for (int i = 0; i < 32; ++i) o[i] *= alpha;
+          tmem_st32(tO + 32 * c, o);
         }
       }
-      // P = exp2(s * scale - m_run) -> bf16 in the 128-byte swizzled K-major layout of
-      // the P V operand; the row sum uses 8 independent partial sums.
+      // P = exp2(s * scale - m_run) as bf16 pairs into the first 64 columns of S_i
       const float neg_m = -m_run;
       float ps[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) ps[i] = 0.f;
 #pragma unroll
-      for (int c = 0; c < kBN / 8; ++c) {
-        float e[8];
+      for (int h = 0; h < 2; ++h) {
+        uint32_t pk[32];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          e[i] = fast_exp2(fmaf(s[c * 8 + i], sl2, neg_m));
-          ps[i] += e[i];
+        for (int c = 0; c < 32; ++c) {
+          const float e0 = fast_exp2(fmaf(s[64 * h + 2 * c], sl2, neg_m));
+          const float e1 = fast_exp2(fmaf(s[64 * h + 2 * c + 1], sl2, neg_m));
+          ps[(2 * c) & 7] += e0;
+          ps[(2 * c + 1) & 7] += e1;
+          pk[c] = pack_bf16x2(e0, e1);
         }
-        const int panel = c >> 3, chunk = c & 7;
-        uint8_t* dst = sP + panel * (kBM * 128) + r * 128 + ((chunk ^ (r & 7)) << 4);
-        *reinterpret_cast<uint4*>(dst) = pack_bf16x8(e);
+        tmem_st32u(tS + 32 * h, pk);
       }
       l_run += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
-      fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(p_full);
+      mbar_arrive(&p_full[tile]);
     }
     if (!failed) {
-      const bool ok = mbar_wait(o_done, (nkv - 1) & 1, p.err);
+      const bool ok = mbar_wait(&o_done[tile], 0, p.err);
       if (!__all_sync(0xffffffffu, ok)) {
         failed = true;
       } else {
         tc_fence_after();
         const float inv = 1.f / l_run;
-        float o[DH];
-        if constexpr (DH == 128) tmem_ld128(tmem_o + lane_addr, o); else tmem_ld64(tmem_o + lane_addr, o);
-        if (q_row < p.n_q) {
-          bf16* dst = p.out + static_cast<long long>(q_row) * p.ldo + head * DH;
+        bf16* dst = p.out + static_cast<long long>(q_row) * p.ldo + head * DH;
 #pragma unroll
-          for (int c = 0; c < DH / 8; ++c) {
-            float f[8];
+        for (int c = 0; c < DH / 32; ++c) {
+          float o[32];
+          tmem_ld32(tO + 32 * c, o);
+          if (q_row < p.n_q) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) f[i] = o[8 * c + i] * inv;
-            *reinterpret_cast<uint4*>(dst + 8 * c) = pack_bf16x8(f);
+            for (int q = 0; q < 4; ++q) {
+              float f[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) f[i] = o[8 * q + i] * inv;
+              *reinterpret_cast<uint4*>(dst + 32 * c + 8 * q) = pack_bf16x8(f);
+            }
           }
         }
       }
@@ -272,7 +295,7 @@ cudaError_t attention_prepare() {
 
 cudaError_t launch_attention(const AttnArgs& a, int head_dim, cudaStream_t s) {
   if (a.n_q <= 0 || a.n_kv <= 0 || a.n_heads <= 0) return cudaSuccess;
-  dim3 grid((a.n_q + kBM - 1) / kBM, a.n_heads);
+  dim3 grid((a.n_q + 2 * kBM - 1) / (2 * kBM), a.n_heads);
   if (head_dim == 128) {
     attn_fwd_tcgen05<128><<<grid, kThreads, AttnLayout<128>::kSmem, s>>>(a);
   } else if (head_dim == 64) {
