@@ -122,26 +122,35 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
     if (lane == 0) {
       constexpr uint32_t idesc_s = idesc_bf16(kBM, kBN);
       constexpr uint32_t idesc_o = idesc_bf16(kBM, DH);
-      const uint32_t q0 = smem_u32(sQ);
+      // Descriptors are built once: the issue loop only adds constant offsets (the start
+      // address field holds address >> 4), which keeps this thread's issue rate at the
+      // tensor pipe's rate.
+      const uint64_t dq = sw128_desc(smem_u32(sQ));
+      const uint64_t dk = sw128_desc(smem_u32(sK));
+      const uint64_t dv = sw128_desc(smem_u32(sV));
       // S_i(j) = Q_i K_j^T into S_i's TMEM columns
       auto issue_s = [&](int i, int j) {
-        const uint32_t k0 = smem_u32(sK + (j & 1) * L::kKBytes);
-        const uint32_t qi = q0 + i * L::kQBytes;
+        const uint64_t a = dq + static_cast<uint64_t>(i * (L::kQBytes >> 4));
+        const uint64_t b = dk + static_cast<uint64_t>((j & 1) * (L::kKBytes >> 4));
+        const uint32_t d = tmem + i * kBN;
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint32_t off = (kk / 4) * (kBM * 128) + (kk % 4) * 32;
-          umma_bf16(tmem + i * kBN, sw128_desc(qi + off), sw128_desc(k0 + off), idesc_s, kk != 0);
+          constexpr uint32_t panel = (kBM * 128) >> 4;
+          const uint64_t off = (kk / 4) * panel + (kk % 4) * 2;
+          umma_bf16(d, a + off, b + off, idesc_s, kk != 0);
         }
         umma_commit(&s_full[i]);
       };
       // O_i += P_i(j) V_j with P_i read from the first 64 columns of S_i
       auto issue_pv = [&](int i, int j) {
-        const uint32_t v0 = smem_u32(sV + (j & 1) * L::kVBytes);
+        const uint64_t b = dv + static_cast<uint64_t>((j & 1) * (L::kVBytes >> 4));
+        const uint32_t d = tmem + 256 + i * 128, a = tmem + i * kBN;
+        const uint32_t first = j != 0;
 #pragma unroll
         for (int kk = 0; kk < kBN / 16; ++kk) {
-          const uint32_t offv = (kk / 4) * (DH * 128) + (kk % 4) * 32;
-          umma_bf16_tmem_a(tmem + 256 + i * 128, tmem + i * kBN + kk * 8, sw128_desc(v0 + offv), idesc_o,
-                           (j | kk) != 0);
+          constexpr uint32_t panel = (DH * 128) >> 4;
+          const uint64_t offv = (kk / 4) * panel + (kk % 4) * 2;
+          umma_bf16_tmem_a(d, a + kk * 8, b + offv, idesc_o, kk == 0 ? first : 1u);
         }
       };
       do {

@@ -209,6 +209,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __gri
   } else if (warp == 1) {
     if (lane == 0 && kb > 0) {
       constexpr uint32_t idesc = idesc_bf16(kGemmBM, kGemmBN);
+      // descriptors built once: stages and K slices only add offsets to the start
+      // address field (address >> 4), which keeps this thread's issue rate at the tensor
+      // pipe's rate
+      const uint64_t da = sw128_desc(smem_u32(sA)), db = sw128_desc(smem_u32(sB));
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -220,11 +224,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __gri
         for (int k = 0; k < kb; ++k) {
           if (!mbar_wait(&full[stage], phase, p.err)) { failed = true; break; }
           tc_fence_after();
-          const uint32_t a0 = smem_u32(sA + stage * kGemmABytes);
-          const uint32_t b0 = smem_u32(sB + stage * kGemmBBytes);
+          const uint64_t a0 = da + static_cast<uint64_t>(stage * (kGemmABytes >> 4));
+          const uint64_t b0 = db + static_cast<uint64_t>(stage * (kGemmBBytes >> 4));
 #pragma unroll
           for (int kk = 0; kk < kGemmBK / 16; ++kk)
-            umma_bf16(d_tmem, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), idesc, (k | kk) != 0);
+            umma_bf16(d_tmem, a0 + kk * 2, b0 + kk * 2, idesc, kk == 0 ? (k != 0) : 1u);
           umma_commit(&empty[stage]);
           if (++stage == kGemmStages) { stage = 0; phase ^= 1; }
         }
