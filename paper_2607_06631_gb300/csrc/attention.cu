@@ -211,13 +211,15 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
         for (int i = 0; i < kBN; ++i)
           if (i >= valid) s[i] = -INFINITY;
       }
+      // row max: 8 independent chains of three-input maxima
       float pm[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) pm[i] = s[i];
 #pragma unroll
-      for (int i = 8; i < kBN; ++i) pm[i & 7] = fmaxf(pm[i & 7], s[i]);
-      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * sl2;
+      for (int i = 8; i < kBN; i += 16)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
+      const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])) * sl2;
       const bool move = mx > m_run + kRescaleThreshold;
       if (j == 0) {
         m_run = mx;
@@ -235,7 +237,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
           tmem_st32(tO + 32 * c, o);
         }
       }
-      // P = exp2(s * scale - m_run) as bf16 pairs into the first 64 columns of S_i
+      // P = exp2(s * scale - m_run) as bf16 pairs into the first 64 columns of S_i;
+      // scale-and-shift and the row-sum partials run as packed pairs
       const float neg_m = -m_run;
       float ps[8];
 #pragma unroll
@@ -245,10 +248,11 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
         uint32_t pk[32];
 #pragma unroll
         for (int c = 0; c < 32; ++c) {
-          const float e0 = fast_exp2(fmaf(s[64 * h + 2 * c], sl2, neg_m));
-          const float e1 = fast_exp2(fmaf(s[64 * h + 2 * c + 1], sl2, neg_m));
-          ps[(2 * c) & 7] += e0;
-          ps[(2 * c + 1) & 7] += e1;
+          float x0, x1;
+          ffma2(x0, x1, s[64 * h + 2 * c], s[64 * h + 2 * c + 1], sl2, sl2, neg_m, neg_m);
+          const float e0 = fast_exp2(x0);
+          const float e1 = fast_exp2(x1);
+          fadd2(ps[2 * (c & 3)], ps[2 * (c & 3) + 1], e0, e1);
           pk[c] = pack_bf16x2(e0, e1);
         }
         tmem_st32u(tS + 32 * h, pk);
