@@ -166,23 +166,28 @@ struct QkParams {
   RopeTables t;
 };
 
-__global__ void __launch_bounds__(kQkThreads) qk_norm_rope_kernel(const QkParams p) {
+// One CTA per token row.  The row stays in registers as raw bf16 vectors (VPT 16-byte
+// vectors per thread), so several rows per SM are in flight at once.
+template <int VPT>
+__global__ void __launch_bounds__(kQkThreads, 4) qk_norm_rope_kernel(const QkParams p) {
   __shared__ float red[32];
   const long long row = blockIdx.x;
   bf16* base = p.buf + row * p.ld;
   const int nvq = p.nq >> 3, nv = (p.nq + p.nk) >> 3;
   const int vph = p.head_dim >> 3;  // vectors per head (8 or 16); divides 32
-  float v[kQkMaxVec][8];
+  uint4 raw[VPT];
+  float hs[VPT];
   float sq = 0.f, sk = 0.f;
-  float hs[kQkMaxVec];
 #pragma unroll
-  for (int k = 0; k < kQkMaxVec; ++k) {
+  for (int k = 0; k < VPT; ++k) {
     const int c = threadIdx.x + k * kQkThreads;
     float ss = 0.f;
     if (c < nv) {
-      unpack_bf16x8(reinterpret_cast<const uint4*>(base)[c], v[k]);
+      raw[k] = reinterpret_cast<const uint4*>(base)[c];
+      float v[8];
+      unpack_bf16x8(raw[k], v);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) ss += v[k][i] * v[k][i];
+      for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
       if (c < nvq) sq += ss; else sk += ss;
     }
     hs[k] = ss;
@@ -196,7 +201,7 @@ __global__ void __launch_bounds__(kQkThreads) qk_norm_rope_kernel(const QkParams
   } else {
     // per head: the vph threads holding one head are consecutive lanes of one warp
 #pragma unroll
-    for (int k = 0; k < kQkMaxVec; ++k) {
+    for (int k = 0; k < VPT; ++k) {
       float t = hs[k];
       for (int o = vph >> 1; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
       hs[k] = rsqrtf(t / p.head_dim + p.eps);
@@ -211,17 +216,17 @@ __global__ void __launch_bounds__(kQkThreads) qk_norm_rope_kernel(const QkParams
     xx = rem - yy * p.t.grid_w;
   }
 #pragma unroll
-  for (int k = 0; k < kQkMaxVec; ++k) {
+  for (int k = 0; k < VPT; ++k) {
     const int c = threadIdx.x + k * kQkThreads;
     if (c < nv) {
       const bool is_q = c < nvq;
       const int ch0 = (is_q ? c : c - nvq) * 8;  // channel within the q or k part
       const float r = p.mode == 0 ? (is_q ? rq : rk) : hs[k];
-      float g[8];
-      unpack_bf16x8(reinterpret_cast<const uint4*>(is_q ? p.gq : p.gk)[ch0 >> 3], g);
-      float o[8];
+      float v[8], g[8], o[8];
+      unpack_bf16x8(raw[k], v);
+      unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(is_q ? p.gq : p.gk) + (ch0 >> 3)), g);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) o[i] = v[k][i] * r * g[i];
+      for (int i = 0; i < 8; ++i) o[i] = v[i] * r * g[i];
       if (p.rope) {
         const int j0 = (ch0 % p.head_dim) >> 1;  // first rotation pair of this vector
 #pragma unroll
@@ -229,16 +234,16 @@ __global__ void __launch_bounds__(kQkThreads) qk_norm_rope_kernel(const QkParams
           const int j = j0 + i;
           float cs, sn;
           if (j < p.t.p_t) {
-            cs = p.t.cos_t[f * p.t.p_t + j];
-            sn = p.t.sin_t[f * p.t.p_t + j];
+            cs = __ldg(p.t.cos_t + f * p.t.p_t + j);
+            sn = __ldg(p.t.sin_t + f * p.t.p_t + j);
           } else if (j < p.t.p_t + p.t.p_h) {
             const int jj = j - p.t.p_t;
-            cs = p.t.cos_h[yy * p.t.p_h + jj];
-            sn = p.t.sin_h[yy * p.t.p_h + jj];
+            cs = __ldg(p.t.cos_h + yy * p.t.p_h + jj);
+            sn = __ldg(p.t.sin_h + yy * p.t.p_h + jj);
           } else {
             const int jj = j - p.t.p_t - p.t.p_h;
-            cs = p.t.cos_w[xx * p.t.p_w + jj];
-            sn = p.t.sin_w[xx * p.t.p_w + jj];
+            cs = __ldg(p.t.cos_w + xx * p.t.p_w + jj);
+            sn = __ldg(p.t.sin_w + xx * p.t.p_w + jj);
           }
           const float a = o[2 * i], b = o[2 * i + 1];
           o[2 * i] = a * cs - b * sn;
@@ -350,7 +355,11 @@ cudaError_t launch_qk_norm_rope(bf16* buf, long long ld, int rows, int nq, int n
   p.head_dim = head_dim; p.mode = mode; p.eps = eps;
   p.rope = rope != nullptr;
   if (rope) p.t = *rope; else memset(&p.t, 0, sizeof(p.t));
-  qk_norm_rope_kernel<<<rows, kQkThreads, 0, s>>>(p);
+  const int vpt = ((nq + nk) / 8 + kQkThreads - 1) / kQkThreads;
+  if (vpt <= 1) qk_norm_rope_kernel<1><<<rows, kQkThreads, 0, s>>>(p);
+  else if (vpt <= 2) qk_norm_rope_kernel<2><<<rows, kQkThreads, 0, s>>>(p);
+  else if (vpt <= 4) qk_norm_rope_kernel<4><<<rows, kQkThreads, 0, s>>>(p);
+  else qk_norm_rope_kernel<8><<<rows, kQkThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 
