@@ -387,10 +387,14 @@ def run_ours(args):
     dk = kernels[dom]
     traffic = None
     tfile = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tfile):
+    if os.path.exists(tfile) and args.grid is None:
         tr = json.load(open(tfile)).get(args.config, {}).get(dom)
         if tr:
-            traffic = tr
+            import hashlib
+            src = os.path.join(ROOT, tr["source"])
+            sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] if os.path.exists(src) else None
+            if sha == tr["source_sha"]:  # counters taken on this very kernel source
+                traffic = tr["bytes_per_launch"]
     roofline = {"kernel": dom, "bound": dk["bound"], "achieved": dk["achieved"], "peak": dk["peak"],
                 "unit": dk["unit"], "frac": dk["frac"], "traffic": traffic,
                 "peak_source": "%s (%s)" % (peak_src, "bf16_tflops_sustained" if dk["bound"] == "tensor"
