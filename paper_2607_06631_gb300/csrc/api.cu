@@ -394,10 +394,11 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     S.g_o.out = P->x1; S.g_o.ldo = d; S.g_o.out_f32 = 1; S.g_o.ldr = d; S.g_o.res_f32 = 0;
     dfs::AttnArgs& A = S.a_self;
     memset(&A, 0, sizeof(A));
+    // a CTA pair of the attention kernel loads 64-key halves of K and DH/2-row halves of V^T
     if (!make_map(&A.tma_q, P->qk, 2LL * hd, N, 2LL * hd, 64, 128) ||
-        !make_map(&A.tma_vt, P->vt, N, hd, P->vt_ld, 64, dh))
+        !make_map(&A.tma_k, P->qk, 2LL * hd, N, 2LL * hd, 64, 64) ||
+        !make_map(&A.tma_vt, P->vt, N, hd, P->vt_ld, 64, dh / 2))
       return fail(DFS_ECUDA, "tensor map (attention) failed");
-    A.tma_k = A.tma_q;
     A.n_q = N; A.n_kv = N; A.n_heads = S.h_s; A.q_col0 = 0; A.k_col0 = hd;
     A.out = P->attn; A.ldo = hd; A.scale_log2 = scale_log2; A.err = P->err;
   }
@@ -434,8 +435,8 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     S.g_co.res_f32 = 1; S.g_co.gate = nullptr;
     dfs::AttnArgs& A = S.a_cross;
     memset(&A, 0, sizeof(A));
-    if (!make_map(&A.tma_q, P->qc, hcd, N, hcd, 64, 128) || !make_map(&A.tma_k, S.kc, hcd, c.ctx_len, hcd, 64, 128) ||
-        !make_map(&A.tma_vt, S.vct, c.ctx_len, hcd, P->ctx_ld, 64, dh))
+    if (!make_map(&A.tma_q, P->qc, hcd, N, hcd, 64, 128) || !make_map(&A.tma_k, S.kc, hcd, c.ctx_len, hcd, 64, 64) ||
+        !make_map(&A.tma_vt, S.vct, c.ctx_len, hcd, P->ctx_ld, 64, dh / 2))
       return fail(DFS_ECUDA, "tensor map (cross attention) failed");
     A.n_q = N; A.n_kv = c.ctx_len; A.n_heads = S.hc; A.q_col0 = 0; A.k_col0 = 0;
     A.out = P->attn; A.ldo = hcd; A.scale_log2 = scale_log2; A.err = P->err;
@@ -924,9 +925,9 @@ dfs_status noalloc_forward(dfs_plan* P, int s, int l, const bf16* x, const bf16*
     DFS_CK(dfs::launch_qk_norm_rope(qk, 2 * hd, N, static_cast<int>(hd), static_cast<int>(hd), S.P[2].p,
                                     S.P[3].p, dh, c.qk_norm_mode, c.ln_eps, &P->rope, st));
     dfs::AttnArgs a = S.a_self;
-    if (!make_map(&a.tma_q, qk, 2 * hd, N, 2 * hd, 64, 128) || !make_map(&a.tma_vt, vt, N, hd, vt_ld, 64, dh))
+    if (!make_map(&a.tma_q, qk, 2 * hd, N, 2 * hd, 64, 128) || !make_map(&a.tma_k, qk, 2 * hd, N, 2 * hd, 64, 64) ||
+        !make_map(&a.tma_vt, vt, N, hd, vt_ld, 64, dh / 2))
       return fail(DFS_ECUDA, "tensor map (attention) failed");
-    a.tma_k = a.tma_q;
     a.out = attn;
     DFS_CK(dfs::launch_attention(a, dh, st));
     dfs::GemmArgs o = S.g_o;

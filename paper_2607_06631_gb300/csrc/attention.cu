@@ -1,20 +1,24 @@
-// K5: non-causal flash attention over the retained heads only, on tcgen05 tensor cores.
+// K5: non-causal flash attention over the retained heads only, on tcgen05 tensor cores,
+// with CTA pairs (a cluster of 2 CTAs on two SMs) issuing 2-SM MMAs.
 //
-// One CTA = two 128-row query tiles (Q0, Q1) of one head, sharing every key / value
-// tile.  Per key / value block j of 128 tokens and tile i:
-//   S_i = Q_i K_j^T      tcgen05.mma (M=128, N=128, K=DH), fp32 into TMEM
-//   P_i = exp2(S_i * scale - m_i)   softmax warpgroup i (thread = query row), bf16 written
-//                        back into the first 64 columns of S_i's TMEM region
-//   O_i += P_i V_j       tcgen05.mma with A read from TMEM (M=128, N=DH, K=128)
-// The single MMA thread issues  S0_j, PV1_{j-1}, S1_j, PV0_j, S0_{j+1}, PV1_j, ...  so the
-// softmax of one tile runs while the tensor core works on the other tile (a window of two
-// 128x128x128 MMAs).  V arrives pre-transposed (V^T [heads*DH, n_kv], written by the QKV
-// projection's epilogue) so every shared-memory operand is K-major.  The running max only
-// moves when it grows by more than 2^8 (exact: the same stale max enters O and the row
-// sum); O is then rescaled in TMEM.  K and V sit in separate two-deep rings.
+// A CTA pair covers 512 query rows of one head: CTA r (r = 0, 1 in the pair) owns rows
+// [512 c + 256 r, +256) as two 128-row tiles.  Tile i of both CTAs forms one M = 256 MMA:
+//   S_i = Q_i K_j^T      tcgen05.mma.cta_group::2 (M=256, N=128, K=DH) -> each CTA's TMEM
+//   P_i = exp2(S_i * scale - m_i)   softmax warpgroup i of each CTA (thread = query row),
+//                        bf16 written back into the first 64 columns of S_i's TMEM region
+//   O_i += P_i V_j       tcgen05.mma.cta_group::2 with A read from both CTAs' TMEM
+// For each 2-SM MMA each CTA holds only half of the B operand: keys [64 r, 64 r + 64) of K_j
+// and V^T rows [DH/2 r, DH/2 r + DH/2), so every SM reads half as many operand bytes from
+// shared memory and loads half of each K/V tile from L2.  The even CTA's single MMA thread
+// issues  S0_j, PV1_{j-1}, S1_j, PV0_j, S0_{j+1}, PV1_j, ...  so either tile's softmax overlaps
+// two MMAs of the other tile; its commits are multicast to both CTAs' barriers.  Both CTAs'
+// TMA loads complete on the even CTA's barriers.  V arrives pre-transposed (V^T written by
+// the QKV projection's epilogue) so every shared-memory operand is K-major.  The running max
+// only moves when it grows by more than 2^8 (exact: the same stale max enters O and the row
+// sum); O is then rescaled in TMEM.
 //
-//   warp 0      TMA: Q0, Q1 once; K_j and V^T_j into their rings
-//   warp 1      MMA issuer (single thread) + TMEM owner (512 columns: S0, S1, O0, O1)
+//   warp 0      TMA: own Q0, Q1 once; own halves of K_j and V^T_j into three-deep rings
+//   warp 1      TMEM allocation (collective over the pair); in the even CTA also the MMA thread
 //   warps 2..5  softmax / rescale / output of tile 0
 //   warps 6..9  softmax / rescale / output of tile 1
 #include "kernels.cuh"
@@ -22,64 +26,154 @@
 namespace dfs {
 namespace {
 
-constexpr int kBM = 128;   // query rows per tile (two tiles per CTA)
+constexpr int kBM = 128;   // query rows per tile (two tiles per CTA, four per pair)
 constexpr int kBN = 128;   // key / value rows per block
+constexpr int kStages = 3; // K and V ring depth
 constexpr int kThreads = 320;
 constexpr float kRescaleThreshold = 8.f;  // log2 units
 
 template <int DH>
 struct AttnLayout {
-  static constexpr int kQBytes = kBM * DH * 2;   // one query tile
-  static constexpr int kKBytes = kBN * DH * 2;   // one key tile
-  static constexpr int kVBytes = DH * kBN * 2;   // one V^T tile
-  static constexpr int kSmem = 2 * kQBytes + 2 * kKBytes + 2 * kVBytes + 1024 + 256;
-  static constexpr uint32_t kTmemCols = 512;     // S0 [0,128) S1 [128,256) O0 [256,..) O1 [384,..)
+  static constexpr int kQBytes = kBM * DH * 2;          // one query tile
+  static constexpr int kKBytes = (kBN / 2) * DH * 2;    // this CTA's half of a key tile
+  static constexpr int kVBytes = (DH / 2) * kBN * 2;    // this CTA's half of a V^T tile
+  static constexpr int kKPanel = (kBN / 2) * 128;       // bytes per 64-wide K panel
+  static constexpr int kVPanel = (DH / 2) * 128;        // bytes per 64-wide V^T panel
+  static constexpr int kSmemUsed = 2 * kQBytes + kStages * (kKBytes + kVBytes) + 1024 + 256;
+  // at least 120 KB so that a second CTA can never share the SM: two pairs interleaved over
+  // the same two SMs could otherwise each hold one SM's TMEM while waiting for the other's
+  static constexpr int kSmem = kSmemUsed < 120 * 1024 ? 120 * 1024 : kSmemUsed;
+  static constexpr uint32_t kTmemCols = 512;            // S0 [0,128) S1 [128,256) O0 [256,..) O1 [384,..)
 };
 
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+// Shared-memory address of the same object in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_to_rank(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// 2D tile load into this CTA's shared memory whose completion is counted on an mbarrier
+// of the pair's even CTA (`bar` is a shared::cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];"
+      ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
+      : "memory");
+}
+
+// Bounded wait with cluster-scope acquire (arrivals may come from the peer CTA).
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, int* err) {
+  const uint32_t a = smem_u32(bar);
+  long long t0 = 0;
+  for (uint32_t n = 0;; ++n) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(a), "r"(parity)
+        : "memory");
+    if (ok) return true;
+    if (n == 0) t0 = clock64();
+    if ((n & 127u) == 127u) {
+      if (*reinterpret_cast<volatile int*>(err) != kErrNone) return false;
+      if (clock64() - t0 > kWaitCycles) {
+        atomicExch(err, kErrTimeout);
+        return false;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void mma_pair_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_pair_ts(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d),
+      "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
+// Arrives once on `bar` (same shared-memory offset) in both CTAs of the pair when every
+// MMA issued so far by this thread has completed.
+__device__ __forceinline__ void commit_pair(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          smem_u32(bar)),
+      "h"(static_cast<unsigned short>(3))
+      : "memory");
+}
+
 template <int DH>
-__global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_constant__ AttnArgs p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    attn_fwd_tcgen05(const __grid_constant__ AttnArgs p) {
   using L = AttnLayout<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;                        // tile i at i * kQBytes
-  uint8_t* sK = sQ + 2 * L::kQBytes;         // ring slot b at b * kKBytes
-  uint8_t* sV = sK + 2 * L::kKBytes;         // ring slot b at b * kVBytes
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + 2 * L::kVBytes);
-  uint64_t* q_full = bars;                   // 1
-  uint64_t* k_full = bars + 1;               // [2]
-  uint64_t* k_empty = k_full + 2;            // [2]
-  uint64_t* v_full = k_empty + 2;            // [2]
-  uint64_t* v_empty = v_full + 2;            // [2]
-  uint64_t* s_full = v_empty + 2;            // [2] per tile: S_i of the current block ready
-  uint64_t* p_full = s_full + 2;             // [2] per tile: P_i written (and O_i rescaled)
+  uint8_t* sK = sQ + 2 * L::kQBytes;         // ring slot s at s * kKBytes
+  uint8_t* sV = sK + kStages * L::kKBytes;   // ring slot s at s * kVBytes
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + kStages * L::kVBytes);
+  uint64_t* q_full = bars;                   // 1   (even CTA's copy counts both CTAs' bytes)
+  uint64_t* k_full = bars + 1;               // [kStages]
+  uint64_t* k_empty = k_full + kStages;      // [kStages]
+  uint64_t* v_full = k_empty + kStages;      // [kStages]
+  uint64_t* v_empty = v_full + kStages;      // [kStages]
+  uint64_t* s_full = v_empty + kStages;      // [2] per tile: S_i of the current block ready
+  uint64_t* p_full = s_full + 2;             // [2] per tile: P_i written by all 8 warps of the pair
   uint64_t* o_done = p_full + 2;             // [2] per tile: last P_i V accumulated
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_done + 2);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
   const int head = blockIdx.y;
-  const int q_base = blockIdx.x * (2 * kBM);
+  const int q_base = (blockIdx.x >> 1) * (4 * kBM) + static_cast<int>(rank) * (2 * kBM);
   const int nkv = (p.n_kv + kBN - 1) / kBN;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&k_full[b], 1);
-      mbar_init(&k_empty[b], 1);
-      mbar_init(&v_full[b], 1);
-      mbar_init(&v_empty[b], 1);
       mbar_init(&s_full[b], 1);
-      mbar_init(&p_full[b], 128);
+      mbar_init(&p_full[b], 8);
       mbar_init(&o_done[b], 1);
     }
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, L::kTmemCols);
-    tmem_relinquish();
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(L::kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // both CTAs' barriers are initialised before any cross-CTA traffic
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   bool failed = false;
@@ -91,99 +185,106 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
       tma_prefetch_desc(&p.tma_vt);
       const int qx = p.q_col0 + head * DH;
       const int kx = p.k_col0 + head * DH;
-      mbar_arrive_expect_tx(q_full, 2 * L::kQBytes);
+      const uint32_t lq = map_to_rank(q_full, 0);
+      if (rank == 0) mbar_arrive_expect_tx(q_full, 2 * 2 * L::kQBytes);
 #pragma unroll
       for (int i = 0; i < 2; ++i)
 #pragma unroll
         for (int c = 0; c < DH / 64; ++c)
-          tma_load_2d(sQ + i * L::kQBytes + c * (kBM * 128), &p.tma_q, q_full, qx + 64 * c, q_base + i * kBM);
+          tma_load_2d_pair(sQ + i * L::kQBytes + c * (kBM * 128), &p.tma_q, lq, qx + 64 * c, q_base + i * kBM);
       // K runs one block ahead of V: K_j is needed by S0_j long before V_j by PV0_j
       for (int j = 0; j <= nkv && !failed; ++j) {
         if (j < nkv) {
-          const int b = j & 1;
-          if (!mbar_wait(&k_empty[b], ((j >> 1) & 1) ^ 1, p.err)) { failed = true; break; }
-          mbar_arrive_expect_tx(&k_full[b], L::kKBytes);
+          const int s = j % kStages;
+          if (!mbar_wait_cluster(&k_empty[s], ((j / kStages) & 1) ^ 1, p.err)) { failed = true; break; }
+          if (rank == 0) mbar_arrive_expect_tx(&k_full[s], 2 * L::kKBytes);
+          const uint32_t lk = map_to_rank(&k_full[s], 0);
 #pragma unroll
           for (int c = 0; c < DH / 64; ++c)
-            tma_load_2d(sK + b * L::kKBytes + c * (kBN * 128), &p.tma_k, &k_full[b], kx + 64 * c, j * kBN);
+            tma_load_2d_pair(sK + s * L::kKBytes + c * L::kKPanel, &p.tma_k, lk, kx + 64 * c,
+                             j * kBN + static_cast<int>(rank) * (kBN / 2));
         }
         if (j >= 1) {
-          const int jv = j - 1, b = jv & 1;
-          if (!mbar_wait(&v_empty[b], ((jv >> 1) & 1) ^ 1, p.err)) { failed = true; break; }
-          mbar_arrive_expect_tx(&v_full[b], L::kVBytes);
+          const int jv = j - 1, s = jv % kStages;
+          if (!mbar_wait_cluster(&v_empty[s], ((jv / kStages) & 1) ^ 1, p.err)) { failed = true; break; }
+          if (rank == 0) mbar_arrive_expect_tx(&v_full[s], 2 * L::kVBytes);
+          const uint32_t lv = map_to_rank(&v_full[s], 0);
 #pragma unroll
           for (int c = 0; c < kBN / 64; ++c)
-            tma_load_2d(sV + b * L::kVBytes + c * (DH * 128), &p.tma_vt, &v_full[b], jv * kBN + 64 * c,
-                        head * DH);
+            tma_load_2d_pair(sV + s * L::kVBytes + c * L::kVPanel, &p.tma_vt, lv, jv * kBN + 64 * c,
+                             head * DH + static_cast<int>(rank) * (DH / 2));
         }
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t idesc_s = idesc_bf16(kBM, kBN);
-      constexpr uint32_t idesc_o = idesc_bf16(kBM, DH);
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16(2 * kBM, kBN);
+      constexpr uint32_t idesc_o = idesc_bf16(2 * kBM, DH);
       // Descriptors are built once: the issue loop only adds constant offsets (the start
       // address field holds address >> 4), which keeps this thread's issue rate at the
       // tensor pipe's rate.
       const uint64_t dq = sw128_desc(smem_u32(sQ));
       const uint64_t dk = sw128_desc(smem_u32(sK));
       const uint64_t dv = sw128_desc(smem_u32(sV));
-      // S_i(j) = Q_i K_j^T into S_i's TMEM columns
+      // S_i(j) = Q_i K_j^T into S_i's TMEM columns of both CTAs
       auto issue_s = [&](int i, int j) {
         const uint64_t a = dq + static_cast<uint64_t>(i * (L::kQBytes >> 4));
-        const uint64_t b = dk + static_cast<uint64_t>((j & 1) * (L::kKBytes >> 4));
+        const uint64_t b = dk + static_cast<uint64_t>((j % kStages) * (L::kKBytes >> 4));
         const uint32_t d = tmem + i * kBN;
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
-          constexpr uint32_t panel = (kBM * 128) >> 4;
-          const uint64_t off = (kk / 4) * panel + (kk % 4) * 2;
-          umma_bf16(d, a + off, b + off, idesc_s, kk != 0);
+          constexpr uint32_t qpanel = (kBM * 128) >> 4, kpanel = L::kKPanel >> 4;
+          mma_pair_ss(d, a + (kk / 4) * qpanel + (kk % 4) * 2, b + (kk / 4) * kpanel + (kk % 4) * 2, idesc_s,
+                      kk != 0);
         }
-        umma_commit(&s_full[i]);
+        commit_pair(&s_full[i]);
       };
-      // O_i += P_i(j) V_j with P_i read from the first 64 columns of S_i
+      // O_i += P_i(j) V_j with P_i read from the first 64 columns of S_i in both CTAs
       auto issue_pv = [&](int i, int j) {
-        const uint64_t b = dv + static_cast<uint64_t>((j & 1) * (L::kVBytes >> 4));
+        const uint64_t b = dv + static_cast<uint64_t>((j % kStages) * (L::kVBytes >> 4));
         const uint32_t d = tmem + 256 + i * 128, a = tmem + i * kBN;
         const uint32_t first = j != 0;
 #pragma unroll
         for (int kk = 0; kk < kBN / 16; ++kk) {
-          constexpr uint32_t panel = (DH * 128) >> 4;
-          const uint64_t offv = (kk / 4) * panel + (kk % 4) * 2;
-          umma_bf16_tmem_a(d, a + kk * 8, b + offv, idesc_o, kk == 0 ? first : 1u);
+          constexpr uint32_t vpanel = L::kVPanel >> 4;
+          mma_pair_ts(d, a + kk * 8, b + (kk / 4) * vpanel + (kk % 4) * 2, idesc_o, kk == 0 ? first : 1u);
         }
       };
       do {
-        if (!mbar_wait(q_full, 0, p.err)) { failed = true; break; }
-        if (!mbar_wait(&k_full[0], 0, p.err)) { failed = true; break; }
+        if (!mbar_wait_cluster(q_full, 0, p.err)) { failed = true; break; }
+        if (!mbar_wait_cluster(&k_full[0], 0, p.err)) { failed = true; break; }
         tc_fence_after();
         issue_s(0, 0);
         issue_s(1, 0);
-        umma_commit(&k_empty[0]);
+        commit_pair(&k_empty[0]);
         for (int j = 0; j < nkv; ++j) {
-          const int b = j & 1;
-          const uint32_t ph = (j >> 1) & 1;
+          const int s = j % kStages;
+          const uint32_t ph = (j / kStages) & 1;
           // PV0_j
-          if (!mbar_wait(&p_full[0], j & 1, p.err) || !mbar_wait(&v_full[b], ph, p.err)) { failed = true; break; }
+          if (!mbar_wait_cluster(&p_full[0], j & 1, p.err) || !mbar_wait_cluster(&v_full[s], ph, p.err)) {
+            failed = true;
+            break;
+          }
           tc_fence_after();
           issue_pv(0, j);
-          if (j + 1 == nkv) umma_commit(&o_done[0]);
+          if (j + 1 == nkv) commit_pair(&o_done[0]);
           // S0_{j+1}
           if (j + 1 < nkv) {
-            if (!mbar_wait(&k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, p.err)) { failed = true; break; }
+            const int s1 = (j + 1) % kStages;
+            if (!mbar_wait_cluster(&k_full[s1], ((j + 1) / kStages) & 1, p.err)) { failed = true; break; }
             tc_fence_after();
             issue_s(0, j + 1);
           }
           // PV1_j
-          if (!mbar_wait(&p_full[1], j & 1, p.err)) { failed = true; break; }
+          if (!mbar_wait_cluster(&p_full[1], j & 1, p.err)) { failed = true; break; }
           tc_fence_after();
           issue_pv(1, j);
-          umma_commit(&v_empty[b]);
-          if (j + 1 == nkv) umma_commit(&o_done[1]);
+          commit_pair(&v_empty[s]);
+          if (j + 1 == nkv) commit_pair(&o_done[1]);
           // S1_{j+1}
           if (j + 1 < nkv) {
             issue_s(1, j + 1);
-            umma_commit(&k_empty[(j + 1) & 1]);
+            commit_pair(&k_empty[(j + 1) % kStages]);
           }
         }
       } while (false);
@@ -196,11 +297,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
     const uint32_t tS = tmem + tile * kBN + lane_addr;
     const uint32_t tO = tmem + 256 + tile * 128 + lane_addr;
     const int q_row = q_base + tile * kBM + r;
+    const uint32_t p_full_leader = map_to_rank(&p_full[tile], 0);
     const float sl2 = p.scale_log2;
     float m_run = -INFINITY;                 // running max of the scaled scores (log2 units)
     float l_run = 0.f;
     for (int j = 0; j < nkv; ++j) {
-      const bool ok = mbar_wait(&s_full[tile], j & 1, p.err);
+      const bool ok = mbar_wait_cluster(&s_full[tile], j & 1, p.err);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
       float s[kBN];
@@ -258,11 +360,19 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
         tmem_st32u(tS + 32 * h, pk);
       }
       l_run += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+      // The TMEM stores of P are complete (tcgen05.wait::st) and ordered before this
+      // thread-sync point by the tcgen05 fence; the MMA thread orders its MMAs after its
+      // wait with tcgen05.fence::after_thread_sync.  One arrival per warp: local in the
+      // even CTA, remote (relaxed, cluster scope) from the odd one.
       tc_fence_before();
-      mbar_arrive(&p_full[tile]);
+      __syncwarp();
+      if (lane == 0) {
+        if (rank == 0) mbar_arrive(&p_full[tile]);
+        else asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(p_full_leader) : "memory");
+      }
     }
     if (!failed) {
-      const bool ok = mbar_wait(&o_done[tile], 0, p.err);
+      const bool ok = mbar_wait_cluster(&o_done[tile], 0, p.err);
       if (!__all_sync(0xffffffffu, ok)) {
         failed = true;
       } else {
@@ -290,10 +400,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_fwd_tcgen05(const __grid_con
   if (failed) drain_after_error();
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, L::kTmemCols);
-  }
+  cluster_sync();  // the even CTA's MMAs read this CTA's shared memory and TMEM until here
+  tc_fence_after();
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(L::kTmemCols) : "memory");
 }
 
 }  // namespace
@@ -308,7 +418,7 @@ cudaError_t attention_prepare() {
 
 cudaError_t launch_attention(const AttnArgs& a, int head_dim, cudaStream_t s) {
   if (a.n_q <= 0 || a.n_kv <= 0 || a.n_heads <= 0) return cudaSuccess;
-  dim3 grid((a.n_q + 2 * kBM - 1) / (2 * kBM), a.n_heads);
+  dim3 grid(2 * ((a.n_q + 4 * kBM - 1) / (4 * kBM)), a.n_heads);
   if (head_dim == 128) {
     attn_fwd_tcgen05<128><<<grid, kThreads, AttnLayout<128>::kSmem, s>>>(a);
   } else if (head_dim == 64) {

@@ -48,8 +48,8 @@ cudaError_t gemm_prepare();  // opts the kernel into its shared-memory size
 // O[q, h*DH : (h+1)*DH] = softmax(Q_h K_h^T / sqrt(DH)) V_h for the retained heads.
 struct AttnArgs {
   CUtensorMap tma_q;   // over the Q source, box {64, 128}
-  CUtensorMap tma_k;   // over the K source, box {64, 128}
-  CUtensorMap tma_vt;  // over V^T [heads*DH, n_kv], box {64, DH}
+  CUtensorMap tma_k;   // over the K source, box {64, 64} (one CTA's half of a 128-key tile)
+  CUtensorMap tma_vt;  // over V^T [heads*DH, n_kv], box {64, DH/2} (one CTA's half)
   int n_q, n_kv, n_heads;
   int q_col0, k_col0;  // column of head 0 in the Q / K sources
   bf16* out;           // [n_q, ldo]
