@@ -383,12 +383,12 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
   CUtensorMap ma, mb;
   const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(dh)));
   if (hd > 0) {
-    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[0].p, d, 3LL * hd, d, 64, 256))
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[0].p, d, 3LL * hd, d, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (QKV) failed");
     S.g_qkv = gemm_args(P, ma, mb, N, 3 * hd, d, dfs::kEpiBias, S.P[1].p);
     S.g_qkv.out = P->qk; S.g_qkv.ldo = 2 * hd; S.g_qkv.split = 2 * hd;
     S.g_qkv.out_t = P->vt; S.g_qkv.ldt = P->vt_ld;
-    if (!make_map(&ma, P->attn, hd, N, hd, 64, 128) || !make_map(&mb, S.P[4].p, hd, d, hd, 64, 256))
+    if (!make_map(&ma, P->attn, hd, N, hd, 64, 128) || !make_map(&mb, S.P[4].p, hd, d, hd, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (O) failed");
     S.g_o = gemm_args(P, ma, mb, N, d, hd, dfs::kEpiGatedRes, C.bo);
     S.g_o.out = P->x1; S.g_o.ldo = d; S.g_o.out_f32 = 1; S.g_o.ldr = d; S.g_o.res_f32 = 0;
@@ -403,11 +403,11 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     A.out = P->attn; A.ldo = hd; A.scale_log2 = scale_log2; A.err = P->err;
   }
   if (fs > 0) {
-    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[5].p, d, fs, d, 64, 256))
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[5].p, d, fs, d, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (up) failed");
     S.g_up = gemm_args(P, ma, mb, N, fs, d, dfs::kEpiBiasGelu, S.P[6].p);
     S.g_up.out = P->h; S.g_up.ldo = fs;
-    if (!make_map(&ma, P->h, fs, N, fs, 64, 128) || !make_map(&mb, S.P[7].p, fs, d, fs, 64, 256))
+    if (!make_map(&ma, P->h, fs, N, fs, 64, 128) || !make_map(&mb, S.P[7].p, fs, d, fs, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (down) failed");
     S.g_down = gemm_args(P, ma, mb, N, d, fs, dfs::kEpiGatedRes, C.bdown);
     S.g_down.ldo = d; S.g_down.out_f32 = 0; S.g_down.res = P->x1; S.g_down.ldr = d; S.g_down.res_f32 = 1;
@@ -417,18 +417,18 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     if ((e = alloc_n(P, &S.kc, static_cast<long long>(c.ctx_len) * hcd)) ||
         (e = alloc_n(P, &S.vct, static_cast<long long>(hcd) * P->ctx_ld)))
       return e;
-    if (!make_map(&ma, ctx, d, c.ctx_len, d, 64, 128) || !make_map(&mb, S.P[10].p, d, 2LL * hcd, d, 64, 256))
+    if (!make_map(&ma, ctx, d, c.ctx_len, d, 64, 128) || !make_map(&mb, S.P[10].p, d, 2LL * hcd, d, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (cross kv) failed");
     dfs::GemmArgs kv = gemm_args(P, ma, mb, c.ctx_len, 2 * hcd, d, dfs::kEpiBias, S.P[11].p);
     kv.out = S.kc; kv.ldo = hcd; kv.split = hcd; kv.out_t = S.vct; kv.ldt = P->ctx_ld;
     DFS_CK(dfs::launch_gemm(kv, P->num_sms, st));
     DFS_CK(dfs::launch_qk_norm_rope(S.kc, hcd, c.ctx_len, 0, hcd, nullptr, S.P[13].p, dh, c.qk_norm_mode,
                                     c.ln_eps, nullptr, st));
-    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[8].p, d, hcd, d, 64, 256))
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[8].p, d, hcd, d, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (cross q) failed");
     S.g_cq = gemm_args(P, ma, mb, N, hcd, d, dfs::kEpiBias, S.P[9].p);
     S.g_cq.out = P->qc; S.g_cq.ldo = hcd;
-    if (!make_map(&ma, P->attn, hcd, N, hcd, 64, 128) || !make_map(&mb, S.P[14].p, hcd, d, hcd, 64, 256))
+    if (!make_map(&ma, P->attn, hcd, N, hcd, 64, 128) || !make_map(&mb, S.P[14].p, hcd, d, hcd, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (cross o) failed");
     S.g_co = gemm_args(P, ma, mb, N, d, hcd, dfs::kEpiGatedRes, C.cbo);
     S.g_co.out = P->x1; S.g_co.ldo = d; S.g_co.out_f32 = 1; S.g_co.res = P->x1; S.g_co.ldr = d;

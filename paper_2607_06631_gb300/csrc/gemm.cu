@@ -1,12 +1,19 @@
 // K4: persistent, warp-specialised tcgen05 GEMM for the block's projections
 // (QKV, attention output, FFN up / down), D = A * B^T with both operands K-major bf16.
 //
-//   warp 0      TMA producer: A tile 128x64 and B tile 256x64 per stage, 4-stage ring.
-//   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=256, K=16) into one of
-//               two TMEM accumulators (2 x 256 fp32 columns), so the epilogue of tile i
-//               overlaps the main loop of tile i+1.
-//   warps 2..5  epilogue: tcgen05.ld 32 columns at a time, fused bias / GELU / gated
-//               residual, predicated stores for the ragged M and N edges.
+// CTA pairs (clusters of 2 CTAs on two SMs) compute 256 x 256 output tiles with 2-SM MMAs
+// (tcgen05.mma.cta_group::2, M=256, N=256, K=16): CTA r holds the A rows [128 r, 128 r + 128)
+// of the tile and the B rows [128 r, 128 r + 128) (half of N), so each SM stages and reads
+// half of the B operand of a 256 x 256 tile from shared memory, and the pair reads each A and
+// B element from L2 once per tile.  Both CTAs' TMA loads complete on the even CTA's
+// barriers; its single MMA thread's commits are multicast to both CTAs.
+//
+//   warp 0      TMA producer: own A rows 128x64 and own B rows 128x64 per stage, 6-stage ring.
+//   warp 1      TMEM allocation (collective over the pair); in the even CTA the MMA thread,
+//               issuing into one of two accumulators (2 x 256 fp32 columns per CTA), so the
+//               epilogue of tile i overlaps the main loop of tile i+1.
+//   warps 2..5  epilogue of this CTA's 128 rows: tcgen05.ld 32 columns at a time, fused bias /
+//               GELU / gated residual, predicated stores for the ragged M and N edges.
 // Ragged K (f_s is a multiple of 8, not of 64) is covered by TMA zero fill.
 #include "kernels.cuh"
 
@@ -149,7 +156,8 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int row, int c
   }
 }
 
-__global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __grid_constant__ GemmArgs p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+    gemm_bf16_tcgen05(const __grid_constant__ GemmArgs p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -162,7 +170,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __gri
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int m_tiles = (p.M + kGemmBM - 1) / kGemmBM;
+  const uint32_t rank = cluster_rank();
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+  const int m_tiles = (p.M + kGemmTileM - 1) / kGemmTileM;
   const int n_tiles = (p.N + kGemmBN - 1) / kGemmBN;
   const int num_tiles = m_tiles * n_tiles;
   const int kb = (p.K + kGemmBK - 1) / kGemmBK;
@@ -174,16 +184,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __gri
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 128);
+      mbar_init(&tempty[a], 8);  // one arrival per epilogue warp of the pair
     }
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // both CTAs' barriers are initialised before any cross-CTA traffic
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   bool failed = false;
@@ -194,21 +207,24 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __gri
       tma_prefetch_desc(&p.tma_b);
       int stage = 0;
       uint32_t phase = 0;
-      for (int tile = blockIdx.x; tile < num_tiles && !failed; tile += gridDim.x) {
+      for (int tile = pair; tile < num_tiles && !failed; tile += n_pairs) {
         int mt, nt;
         tile_coords(tile, m_tiles, n_tiles, mt, nt);
         for (int k = 0; k < kb; ++k) {
-          if (!mbar_wait(&empty[stage], phase ^ 1, p.err)) { failed = true; break; }
-          mbar_arrive_expect_tx(&full[stage], kGemmStageBytes);
-          tma_load_2d(sA + stage * kGemmABytes, &p.tma_a, &full[stage], k * kGemmBK, mt * kGemmBM);
-          tma_load_2d(sB + stage * kGemmBBytes, &p.tma_b, &full[stage], k * kGemmBK, nt * kGemmBN);
+          if (!mbar_wait_cluster(&empty[stage], phase ^ 1, p.err)) { failed = true; break; }
+          if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * kGemmStageBytes);
+          const uint32_t lf = map_to_rank(&full[stage], 0);
+          tma_load_2d_pair(sA + stage * kGemmABytes, &p.tma_a, lf, k * kGemmBK,
+                           mt * kGemmTileM + static_cast<int>(rank) * kGemmBM);
+          tma_load_2d_pair(sB + stage * kGemmBBytes, &p.tma_b, lf, k * kGemmBK,
+                           nt * kGemmBN + static_cast<int>(rank) * kGemmBRows);
           if (++stage == kGemmStages) { stage = 0; phase ^= 1; }
         }
       }
     }
   } else if (warp == 1) {
-    if (lane == 0 && kb > 0) {
-      constexpr uint32_t idesc = idesc_bf16(kGemmBM, kGemmBN);
+    if (lane == 0 && rank == 0 && kb > 0) {
+      constexpr uint32_t idesc = idesc_bf16(kGemmTileM, kGemmBN);
       // descriptors built once: stages and K slices only add offsets to the start
       // address field (address >> 4), which keeps this thread's issue rate at the tensor
       // pipe's rate
@@ -217,39 +233,40 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __gri
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
-      for (int tile = blockIdx.x; tile < num_tiles && !failed; tile += gridDim.x) {
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, p.err)) { failed = true; break; }
+      for (int tile = pair; tile < num_tiles && !failed; tile += n_pairs) {
+        if (!mbar_wait_cluster(&tempty[acc], acc_phase ^ 1, p.err)) { failed = true; break; }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * kGemmBN;
         for (int k = 0; k < kb; ++k) {
-          if (!mbar_wait(&full[stage], phase, p.err)) { failed = true; break; }
+          if (!mbar_wait_cluster(&full[stage], phase, p.err)) { failed = true; break; }
           tc_fence_after();
           const uint64_t a0 = da + static_cast<uint64_t>(stage * (kGemmABytes >> 4));
           const uint64_t b0 = db + static_cast<uint64_t>(stage * (kGemmBBytes >> 4));
 #pragma unroll
           for (int kk = 0; kk < kGemmBK / 16; ++kk)
-            umma_bf16(d_tmem, a0 + kk * 2, b0 + kk * 2, idesc, kk == 0 ? (k != 0) : 1u);
-          umma_commit(&empty[stage]);
+            mma_pair_ss(d_tmem, a0 + kk * 2, b0 + kk * 2, idesc, kk == 0 ? (k != 0) : 1u);
+          commit_pair(&empty[stage]);
           if (++stage == kGemmStages) { stage = 0; phase ^= 1; }
         }
-        umma_commit(&tfull[acc]);
+        commit_pair(&tfull[acc]);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1;
       }
     }
   } else {
     const int sub = warp & 3;  // TMEM lane quarter this warp may access
-    const int r_in_tile = sub * 32 + lane;
+    const int r_in_tile = static_cast<int>(rank) * kGemmBM + sub * 32 + lane;
+    const uint32_t tempty_leader0 = map_to_rank(&tempty[0], 0), tempty_leader1 = map_to_rank(&tempty[1], 0);
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+    for (int tile = pair; tile < num_tiles; tile += n_pairs) {
       int mt, nt;
       tile_coords(tile, m_tiles, n_tiles, mt, nt);
-      const int row = mt * kGemmBM + r_in_tile;
+      const int row = mt * kGemmTileM + r_in_tile;
       if (kb > 0) {
         // every lane waits; the warp leaves together if any lane gave up, so that the
         // warp-collective TMEM loads below are never split
-        const bool ok = mbar_wait(&tfull[acc], acc_phase, p.err);
+        const bool ok = mbar_wait_cluster(&tfull[acc], acc_phase, p.err);
         if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
         tc_fence_after();
       }
@@ -266,8 +283,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __gri
         epilogue_chunk(p, row, col0, v);
       }
       if (kb > 0) {
+        // this accumulator is read out: one arrival per warp on the even CTA's barrier
         tc_fence_before();
-        mbar_arrive(&tempty[acc]);
+        __syncwarp();
+        if (lane == 0) {
+          if (rank == 0)
+            mbar_arrive(&tempty[acc]);
+          else
+            asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(acc ? tempty_leader1 : tempty_leader0)
+                         : "memory");
+        }
       }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
@@ -277,10 +302,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_bf16_tcgen05(const __gri
   if (failed) drain_after_error();
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
-  }
+  cluster_sync();  // the even CTA's MMAs read this CTA's shared memory and TMEM until here
+  tc_fence_after();
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
 }
 
 }  // namespace
@@ -290,12 +315,12 @@ cudaError_t gemm_prepare() {
 }
 
 cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t s) {
-  const int m_tiles = (a.M + kGemmBM - 1) / kGemmBM;
+  const int m_tiles = (a.M + kGemmTileM - 1) / kGemmTileM;
   const int n_tiles = (a.N + kGemmBN - 1) / kGemmBN;
   const int tiles = m_tiles * n_tiles;
   if (tiles == 0) return cudaSuccess;
-  const int grid = tiles < num_sms ? tiles : num_sms;
-  gemm_bf16_tcgen05<<<grid, kGemmThreads, kGemmSmem, s>>>(a);
+  const int pairs = tiles < num_sms / 2 ? tiles : num_sms / 2;
+  gemm_bf16_tcgen05<<<2 * pairs, kGemmThreads, kGemmSmem, s>>>(a);
   return cudaGetLastError();
 }
 

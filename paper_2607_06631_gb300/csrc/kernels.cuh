@@ -15,16 +15,18 @@ enum EpiMode : int {
   kEpiGatedRes = 2,  // out = res + gate * (acc + bias) (res / out bf16 or fp32)
 };
 
-constexpr int kGemmBM = 128, kGemmBN = 256, kGemmBK = 64, kGemmStages = 4;
+// A CTA pair computes a kGemmTileM x kGemmBN output tile; each CTA stages kGemmBM rows of A
+// and kGemmBRows rows of B per K block.
+constexpr int kGemmBM = 128, kGemmTileM = 256, kGemmBN = 256, kGemmBRows = 128, kGemmBK = 64, kGemmStages = 6;
 constexpr int kGemmThreads = 192;
 constexpr int kGemmABytes = kGemmBM * kGemmBK * 2;
-constexpr int kGemmBBytes = kGemmBN * kGemmBK * 2;
+constexpr int kGemmBBytes = kGemmBRows * kGemmBK * 2;
 constexpr int kGemmStageBytes = kGemmABytes + kGemmBBytes;
 constexpr int kGemmSmem = kGemmStages * kGemmStageBytes + 1024 + 256;
 
 struct GemmArgs {
   CUtensorMap tma_a;  // A [M, K], box {64, 128}, 128 B swizzle
-  CUtensorMap tma_b;  // B [N, K], box {64, 256}, 128 B swizzle
+  CUtensorMap tma_b;  // B [N, K], box {64, 128}, 128 B swizzle
   int M, N, K;
   int mode;
   const bf16* bias;  // [N] or null
