@@ -267,6 +267,7 @@ dfs::GemmArgs gemm_args(dfs_plan* P, const CUtensorMap& a, const CUtensorMap& b,
   g.mode = mode;
   g.bias = bias;
   g.split = N;
+  g.group = dfs::gemm_group(K);
   g.err = P->err;
   return g;
 }

@@ -28,10 +28,9 @@ __device__ __forceinline__ float gelu_tanh(float x) {
   return 0.5f * x * (1.f + t);
 }
 
-// Grouped raster: 16 M-tiles share each sweep over N so that concurrent CTAs reuse
-// both operands from L2.
-__device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mt, int& nt) {
-  constexpr int G = 16;
+// Grouped raster: G M-tiles share each sweep over N so that concurrent CTA pairs reuse both
+// operands from L2.
+__device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int G, int& mt, int& nt) {
   const int group = tile / (G * n_tiles);
   const int first_m = group * G;
   const int gsz = min(m_tiles - first_m, G);
@@ -209,7 +208,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       uint32_t phase = 0;
       for (int tile = pair; tile < num_tiles && !failed; tile += n_pairs) {
         int mt, nt;
-        tile_coords(tile, m_tiles, n_tiles, mt, nt);
+        tile_coords(tile, m_tiles, n_tiles, p.group, mt, nt);
         for (int k = 0; k < kb; ++k) {
           if (!mbar_wait_cluster(&empty[stage], phase ^ 1, p.err)) { failed = true; break; }
           if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * kGemmStageBytes);
@@ -261,7 +260,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     uint32_t acc_phase = 0;
     for (int tile = pair; tile < num_tiles; tile += n_pairs) {
       int mt, nt;
-      tile_coords(tile, m_tiles, n_tiles, mt, nt);
+      tile_coords(tile, m_tiles, n_tiles, p.group, mt, nt);
       const int row = mt * kGemmTileM + r_in_tile;
       if (kb > 0) {
         // every lane waits; the warp leaves together if any lane gave up, so that the
