@@ -34,7 +34,7 @@ import synth  # noqa: E402
 
 METRIC = "pruned-block TFLOP/s and % bf16 tensor peak; pruned/dense speedup vs ideal"
 KINDS = ("modulation", "adaln", "gemm_qkv", "qk_norm_rope", "attention", "gemm_o", "gemm_up", "gemm_down",
-         "cross", "other")
+         "cross", "other", "gather")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -109,6 +109,8 @@ def kernel_units(cfg):
         u["adaln"] += N * d * (2 + 2) + N * d * (4 + 2)      # x bf16 -> xm, x1 fp32 -> xm2
         u["qk_norm_rope"] += 2.0 * N * 2 * hd * 2              # q, k read + written
         u["modulation"] += 6.0 * d * d * 2                     # W_t read once
+        if cfg.engine == 1:                                    # union engine: FFN panels gathered
+            u["gather"] += 2.0 * (2 * fs * d * 2)              # W_up_s, W_down_s read + written
         if cfg.has_cross:
             hc = cfg.xheads_kept[s][0] * dh
             u["cross"] += 4.0 * N * d * hc + 4.0 * N * cfg.ctx_len * hc
@@ -311,6 +313,7 @@ def run_ours(args):
     build.build()
     peaks, peak_src = load_peaks()
     cfg = get_config(args.config, args.grid)
+    cfg.engine = dfs.ENGINES[args.engine]
     T, L = cfg.n_steps, cfg.n_layers
     stream = torch.cuda.current_stream()
     if L == 1:
@@ -328,6 +331,7 @@ def run_ours(args):
         prob = None
     out = torch.empty_like(x)
     lat = x.clone()
+    weight_bytes, device_bytes = dfs.dfs_plan_memory(plan)
     flops = [sum(dfs.dfs_plan_flops(plan, s, l) for l in range(L)) for s in range(T)]
     flops_step = sum(flops)
 
@@ -453,7 +457,10 @@ def run_ours(args):
             "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": workload_desc(cfg),
-                       "l2": "inputs larger than L2 (x %.0f MB, per-step weight panels %.0f-%.0f MB); no flush "
+                       "engine": args.engine,
+                       "plan_weight_gb": round(weight_bytes / 1e9, 3),
+                       "plan_device_gb": round(device_bytes / 1e9, 3),
+                       "l2": "inputs larger than L2 (x %.0f MB, per-step weights read %.0f-%.0f MB); no flush "
                              "between steps" % (cfg.n_tokens * cfg.dim * 2 / 1e6, panel_mb(cfg)[0],
                                                 panel_mb(cfg)[1]),
                        "parallelism": "replicas (one independent block per GPU)" if world > 1 else "1 GPU"},
@@ -487,6 +494,9 @@ def main():
                     help="wan14b (default), wan13b, wan14b_cross, sweep720 (keep 1.0..0.5 as six steps), "
                          "sweep720:<ratio>, wan14b_x<L> (L-layer 4-step denoise with cross-attention), tiny")
     ap.add_argument("--grid", default=None, help="override the latent grid T,H,W (smaller profiling cases)")
+    ap.add_argument("--engine", choices=("compacted", "union"), default="compacted",
+                    help="weights per (step, layer) compacted once (default), or one union super-model per "
+                         "layer gathered by the projections' TMA producers (Sec. 4.3)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()

@@ -35,12 +35,27 @@ typedef enum {
   DFS_EUNSUPPORTED = 5   /* valid request this build does not implement                */
 } dfs_status;
 
+/* How a plan holds the weights of the retained units (Sec. 4.3, Fig. 1(c)).
+ *   DFS_ENGINE_COMPACTED: every (step, layer) gets its own dense copy of its retained
+ *     weights, gathered once at plan creation; the projections read them as stored.
+ *     Weight memory: the sum over steps of the retained weights.
+ *   DFS_ENGINE_UNION: the plan keeps one union super-model per layer (the weights of the
+ *     units retained at ANY step, theta_union) plus the per-step index tables I_t.  At every
+ *     forward the head-granular projections (QKV, output, cross-attention Q / output)
+ *     gather the step's heads from the union inside their TMA producer, and the step's FFN
+ *     panels (8-channel chunks) are gathered from the union into one plan-owned scratch
+ *     pair (sized for the largest step) by the compaction kernel.  Weight memory: the union
+ *     plus that scratch.  Results are bit-identical to DFS_ENGINE_COMPACTED (the same
+ *     operands reach the tensor cores in the same order). */
+typedef enum { DFS_ENGINE_COMPACTED = 0, DFS_ENGINE_UNION = 1 } dfs_engine;
+
 /* Block shapes.  N = grid_t * grid_h * grid_w latent tokens (frame-major).
  *   dim = n_heads * head_dim, head_dim in {64, 128}, ffn_dim % ffn_chunk == 0,
  *   ffn_chunk = 8 (App. A), n_steps = 4 (Sec. 3.1; 1..8 accepted).
  *   qk_norm_mode: 0 = QK RMSNorm over the retained q (k) channels of a token row,
  *                 1 = over each head's head_dim channels.
- *   has_cross = 1 adds text cross-attention over ctx_len context tokens (1..4096). */
+ *   has_cross = 1 adds text cross-attention over ctx_len context tokens (1..4096).
+ *   engine: a dfs_engine value. */
 typedef struct {
   int dim, n_heads, head_dim, ffn_dim, ffn_chunk, n_layers, n_steps;
   int grid_t, grid_h, grid_w;
@@ -48,6 +63,7 @@ typedef struct {
   float ln_eps;      /* LayerNorm / RMSNorm epsilon (1e-6)       */
   float rope_theta;  /* 3D RoPE base (1e4)                       */
   int qk_norm_mode;
+  int engine;
 } dfs_config;
 
 /* One layer's full (unpruned) weights; bf16 DEVICE pointers, borrowed for the duration
@@ -73,10 +89,12 @@ typedef struct {
 
 /* Builds a plan (Sec. 4.3: the union super-model plus the per-step index tables I_t).
  * Validates every argument on the host before any CUDA call, builds the ascending
- * retained head / chunk lists per (step, layer), gathers the retained weight slices
- * into dense bf16 panels on the device (one compaction kernel per panel), copies the
- * full bias / modulation vectors, precomputes the RoPE tables and, with has_cross,
- * the context keys / values per (step, layer); allocates the workspace for N tokens.
+ * retained head / chunk lists per (step, layer) and the union lists per layer, gathers
+ * the retained weight slices into dense bf16 panels on the device (per (step, layer)
+ * under DFS_ENGINE_COMPACTED, per layer from the union under DFS_ENGINE_UNION; one
+ * compaction kernel per panel), copies the full bias / modulation vectors, precomputes
+ * the RoPE tables and, with has_cross, the context keys / values per (step, layer);
+ * allocates the workspace for N tokens.
  *   w_t [6*dim, dim], b_t [6*dim]: shared adaLN linear (bf16 device, borrowed).
  *   ctx [ctx_len, dim] bf16 device or NULL when has_cross == 0 (borrowed).
  * Synchronises `stream` before returning.  On failure *out is NULL and everything
@@ -136,8 +154,11 @@ dfs_status dfs_denoise(dfs_plan* plan, void* latents, int n_steps, const void* t
 /* Test hooks ---------------------------------------------------------------------- */
 
 /* Index lists of I_t for (step, layer).  kind: 0 = retained head ids, 1 = retained FFN
- * chunk ids, 2 = retained cross-attention head ids.  Writes *count ids (ascending) to
- * `out` (host, may be NULL to query the count). */
+ * chunk ids, 2 = retained cross-attention head ids; 3, 4, 5 = the ids of the layer's
+ * union super-model (heads / FFN chunks / cross heads retained at any step of the plan,
+ * independent of `step`); 6, 7, 8 = the positions of the step's retained heads / chunks /
+ * cross heads inside that union (ascending; kind 3 indexed by kind 6 gives kind 0).
+ * Writes *count ids to `out` (host, may be NULL to query the count).  Every engine. */
 dfs_status dfs_plan_indices(const dfs_plan* plan, int step, int layer, int kind,
                             int32_t* out, int* count);
 
@@ -146,9 +167,25 @@ dfs_status dfs_plan_indices(const dfs_plan* plan, int step, int layer, int kind,
  * 3 gk [h_s dh], 4 Wo [dim, h_s dh], 5 W_up [f_s, dim], 6 b_up [f_s],
  * 7 W_down [dim, f_s]; cross: 8 cWq [hc dh, dim], 9 cbq, 10 cWkv [2 hc dh, dim],
  * 11 cbkv, 12 cgq, 13 cgk, 14 cWo [dim, hc dh].  A panel with zero rows or columns
- * returns *dev == NULL. */
+ * returns *dev == NULL.  Under DFS_ENGINE_UNION the weight matrices (0, 4, 5, 7, 8, 10,
+ * 14) have no per-step copy: they return their shape with *dev == NULL. */
 dfs_status dfs_plan_panel(const dfs_plan* plan, int step, int layer, int which,
                           const void** dev, int64_t* rows, int64_t* cols, int64_t* ld);
+
+/* Device address and shape of a union panel of `layer` (DFS_ENGINE_UNION only; bf16,
+ * row-major, leading dim *ld).  With nu / nf / nx the union head / chunk / cross-head
+ * counts: which 0 Wqkv [3 nu dh, dim] (the q, k and v rows of the union heads, in that
+ * order), 1 Wo [dim, nu dh], 2 W_up [8 nf, dim], 3 W_down [dim, 8 nf], 4 cWq [nx dh, dim],
+ * 5 cWo [dim, nx dh].  Errors:
+ * DFS_EINVAL, DFS_EUNSUPPORTED for a plan of another engine. */
+dfs_status dfs_plan_union_panel(const dfs_plan* plan, int layer, int which, const void** dev,
+                                int64_t* rows, int64_t* cols, int64_t* ld);
+
+/* Device memory held by the plan: *weight_bytes = its weight copies (compacted panels or
+ * union panels, with the per-step bias / norm-scale vectors), *device_bytes = every device
+ * allocation it owns (weights, workspace including the union engine's FFN scratch,
+ * tables).  Host only. */
+dfs_status dfs_plan_memory(const dfs_plan* plan, int64_t* weight_bytes, int64_t* device_bytes);
 
 /* Algorithmic FLOPs (2 per multiply-add) of one block forward at (step, layer). */
 dfs_status dfs_plan_flops(const dfs_plan* plan, int step, int layer, double* flops);
@@ -185,7 +222,8 @@ typedef enum {
   DFS_K_GEMM_DOWN = 7,    /* FFN down projection + gated residual                      */
   DFS_K_CROSS = 8,        /* every kernel of the cross-attention branch                */
   DFS_K_OTHER = 9,        /* bias-only branches, Euler update, block-gate copies       */
-  DFS_K_COUNT = 10
+  DFS_K_GATHER = 10,      /* union engine: per-forward FFN panel gathers from the union */
+  DFS_K_COUNT = 11
 } dfs_kernel_kind;
 
 /* Per-kernel timing of the forwards enqueued on this plan.  enable = 1 resets the

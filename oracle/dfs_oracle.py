@@ -42,6 +42,7 @@ import numpy as np
 
 __all__ = [
     "gates_from_soft_masks", "ffn_channel_gate", "compact_indices", "compact_panels",
+    "union_tables", "union_panels",
     "linear", "modulation", "layer_norm", "adaln", "rms_norm", "rope_pairs", "rope_angles",
     "apply_rope", "attention", "gelu_tanh", "block_forward_masked",
     "block_forward_compacted", "block_flops", "denoise", "MacCounter",
@@ -127,6 +128,64 @@ def compact_panels(layer_w: Dict[str, np.ndarray], idx: Dict[str, np.ndarray]) -
             "cgq": layer_w["cgq"][xr], "cgk": layer_w["cgk"][xr],
             "cwo": layer_w["cwo"][:, xr],
         })
+    return P
+
+
+def union_tables(cfg, masks, layer: int) -> Dict[str, object]:
+    """The union super-model of one layer and its per-step index tables (Sec. 4.3,
+    Fig. 1(c)): theta_union holds every unit that some step retains, and I_t addresses
+    step t's retained units inside it.
+
+    heads / chunks / xheads: ascending unit ids retained at one step or more (block gates
+    do not enter: a unit belongs to the union as soon as any step's gate keeps it).
+    pos_heads / pos_chunks / pos_xheads: per step, for each retained unit of that step
+    (ascending), its index in the union list.
+    """
+    H = cfg.n_heads
+    hg = np.asarray(masks["head_gate"])[:, layer].astype(bool)
+    fg = np.asarray(masks["ffn_gate"])[:, layer].astype(bool)
+    T = hg.shape[0]
+    out = {"heads": [], "chunks": [], "xheads": [], "pos_heads": [], "pos_chunks": [], "pos_xheads": []}
+    # a unit is in the union iff some step keeps it
+    out["heads"] = np.array([h for h in range(H) if any(hg[s, h] for s in range(T))], dtype=np.int32)
+    out["chunks"] = np.array([k for k in range(fg.shape[1]) if any(fg[s, k] for s in range(T))], dtype=np.int32)
+    if cfg.has_cross:
+        xg = masks.get("xhead_gate")
+        xgl = np.ones((T, H), bool) if xg is None else np.asarray(xg)[:, layer].astype(bool)
+        out["xheads"] = np.array([h for h in range(H) if any(xgl[s, h] for s in range(T))], dtype=np.int32)
+    for s in range(T):
+        idx = compact_indices(cfg, masks, s, layer)
+        where = {u: i for i, u in enumerate(out["heads"])}
+        out["pos_heads"].append(np.array([where[h] for h in idx["heads"]], dtype=np.int32))
+        where = {u: i for i, u in enumerate(out["chunks"])}
+        out["pos_chunks"].append(np.array([where[k] for k in idx["chunks"]], dtype=np.int32))
+        if cfg.has_cross:
+            where = {u: i for i, u in enumerate(out["xheads"])}
+            out["pos_xheads"].append(np.array([where[h] for h in idx["xheads"]], dtype=np.int32))
+    return out
+
+
+def union_panels(cfg, layer_w: Dict[str, np.ndarray], union: Dict[str, object]) -> Dict[str, np.ndarray]:
+    """Weights of the union super-model (Sec. 4.3), gathered from the full layer: the q, k
+    and v rows of the union heads stacked, the matching columns of Wo, the union FFN
+    channels' rows of W_up and columns of W_down, and with cross-attention the union cross
+    heads' rows of cWq and columns of cWo.  Selection only (any dtype)."""
+    dh, C = cfg.head_dim, cfg.ffn_chunk
+    hu = np.asarray(union["heads"], dtype=np.int64)
+    r = (hu[:, None] * dh + np.arange(dh)[None, :]).reshape(-1)
+    cu = np.asarray(union["chunks"], dtype=np.int64)
+    ch = (cu[:, None] * C + np.arange(C)[None, :]).reshape(-1)
+    P = {
+        "wqkv": np.concatenate([layer_w["wq"][r], layer_w["wk"][r], layer_w["wv"][r]], axis=0),
+        "wo": layer_w["wo"][:, r],
+        "w_up": layer_w["w_up"][ch],
+        "w_down": layer_w["w_down"][:, ch],
+    }
+    if cfg.has_cross:
+        xu = np.asarray(union["xheads"], dtype=np.int64)
+        xr = (xu[:, None] * dh + np.arange(dh)[None, :]).reshape(-1)
+        P["cwq"] = layer_w["cwq"][xr]
+        P["cwo"] = layer_w["cwo"][:, xr]
     return P
 
 

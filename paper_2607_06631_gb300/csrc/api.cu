@@ -86,12 +86,22 @@ struct Panel {
 struct StepLayer {
   int h_s = 0, f_s = 0, hc = 0;
   std::vector<int> heads, chunks, xheads;
+  std::vector<int> pos_heads, pos_chunks, pos_xheads;  // positions inside the layer's union
+  int* up_rows_u = nullptr;    // union engine: union W_up rows of the step's FFN channels [f_s]
+  int* down_segs_u = nullptr;  // union engine: union W_down 8-column segments of its chunks [f_s / 8]
   Panel P[15];       // indexed like dfs_plan_panel's `which`
   bf16* kc = nullptr;    // cross-attention context keys, normalised [ctx_len, hc dh]
   bf16* vct = nullptr;   // cross-attention context values, transposed [hc dh, ctx_ld]
   dfs::GemmArgs g_qkv, g_o, g_up, g_down, g_cq, g_co;
   dfs::AttnArgs a_self, a_cross;
   double flops = 0;
+};
+
+// The union super-model of one layer (Sec. 4.3): ids of the units retained at any step and,
+// under DFS_ENGINE_UNION, the weights of exactly those units.
+struct LayerUnion {
+  std::vector<int> heads, chunks, xheads;
+  Panel wqkv, wo, wup, wdown, cwq, cwo;  // indexed like dfs_plan_union_panel's `which`
 };
 
 struct LayerConst {
@@ -109,6 +119,12 @@ struct dfs_plan {
   std::vector<uint8_t> block_gate;
   std::vector<StepLayer> sl;  // [T * L]
   std::vector<LayerConst> lc;
+  std::vector<LayerUnion> lu;  // [L]
+  bool uni = false;            // DFS_ENGINE_UNION
+  bf16* ffn_up_s = nullptr;    // union engine: the forward's FFN panels, gathered from the
+  bf16* ffn_down_s = nullptr;  //   union at every forward ([f_s, d] and [d, f_s], largest step)
+  long long bytes_total = 0, bytes_weights = 0;
+  std::vector<void*> temps;    // device buffers needed only during plan creation
   bf16* w_t = nullptr;
   bf16* b_t = nullptr;
   dfs::RopeTables rope{};
@@ -153,6 +169,7 @@ dfs_status dev_alloc(dfs_plan* P, void** out, size_t bytes) {
     return fail(DFS_ENOMEM, "cudaMalloc(%zu) failed: %s", bytes, cudaGetErrorString(e));
   }
   P->allocs.push_back(*out);
+  P->bytes_total += static_cast<long long>(bytes);
   return DFS_OK;
 }
 
@@ -161,10 +178,35 @@ dfs_status alloc_n(dfs_plan* P, T** out, long long n) {
   return dev_alloc(P, reinterpret_cast<void**>(out), static_cast<size_t>(n) * sizeof(T));
 }
 
+// A weight panel of the plan (counted in bytes_weights).
+dfs_status alloc_weights(dfs_plan* P, bf16** out, long long n) {
+  dfs_status e = alloc_n(P, out, n);
+  if (!e) P->bytes_weights += 2 * n;
+  return e;
+}
+
+// A device buffer freed at the end of plan creation (not counted as held by the plan).
+dfs_status alloc_temp(dfs_plan* P, bf16** out, long long n) {
+  *out = nullptr;
+  ++P->n_alloc;
+  if (P->fault_alloc > 0 && P->n_alloc == P->fault_alloc)
+    return fail(DFS_ENOMEM, "injected allocation failure at allocation %d", P->n_alloc);
+  if (n == 0) return DFS_OK;
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(out), static_cast<size_t>(n) * sizeof(bf16));
+  if (e != cudaSuccess) {
+    *out = nullptr;
+    (void)cudaGetLastError();
+    return fail(DFS_ENOMEM, "cudaMalloc(%lld) failed: %s", 2 * n, cudaGetErrorString(e));
+  }
+  P->temps.push_back(*out);
+  return DFS_OK;
+}
+
 void free_plan(dfs_plan* P) {
   if (!P) return;
   for (cudaEvent_t e : P->ev) cudaEventDestroy(e);
   for (void* p : P->allocs) cudaFree(p);
+  for (void* p : P->temps) cudaFree(p);
   delete P;
 }
 
@@ -227,6 +269,8 @@ dfs_status validate(const dfs_config* c, const dfs_layer_weights* layers, const 
     return fail(DFS_EINVAL, "ctx_len must be a multiple of 8 in 8..4096");
   if (c->has_cross && !ctx) return fail(DFS_EINVAL, "ctx is NULL with has_cross");
   if (c->qk_norm_mode != 0 && c->qk_norm_mode != 1) return fail(DFS_EINVAL, "qk_norm_mode must be 0 or 1");
+  if (c->engine != DFS_ENGINE_COMPACTED && c->engine != DFS_ENGINE_UNION)
+    return fail(DFS_EINVAL, "engine must be DFS_ENGINE_COMPACTED or DFS_ENGINE_UNION");
   if (!(c->ln_eps > 0.f) || !(c->rope_theta > 1.f)) return fail(DFS_EINVAL, "ln_eps / rope_theta out of range");
   if (!layers || !w_t || !b_t || !m) return fail(DFS_EINVAL, "NULL weights or masks");
   for (int l = 0; l < c->n_layers; ++l) {
@@ -281,6 +325,16 @@ dfs_status upload_ints(dfs_plan* P, const std::vector<int>& v, int** out, cudaSt
   return DFS_OK;
 }
 
+// Positions of `ids` (ascending) inside `uni` (ascending, a superset): the I_t table that
+// addresses a step's units inside the union super-model.
+std::vector<int> positions_in(const std::vector<int>& ids, const std::vector<int>& uni) {
+  std::vector<int> pos;
+  pos.reserve(ids.size());
+  for (int id : ids)
+    pos.push_back(static_cast<int>(std::lower_bound(uni.begin(), uni.end(), id) - uni.begin()));
+  return pos;
+}
+
 // Builds the index lists, gathers the panels and prebuilds every kernel argument of
 // one (step, layer).
 dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& w, const dfs_masks* m,
@@ -288,6 +342,8 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
   const dfs_config& c = P->cfg;
   const int d = c.dim, H = c.n_heads, dh = c.head_dim, NC = c.ffn_dim / c.ffn_chunk;
   StepLayer& S = P->sl[s * P->L + l];
+  const LayerUnion& U = P->lu[l];
+  const bool uni = P->uni;
   const long long base = static_cast<long long>(s) * c.n_layers + l;
   for (int h = 0; h < H; ++h)
     if (m->head_gate[base * H + h]) S.heads.push_back(h);
@@ -299,6 +355,9 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
   S.h_s = static_cast<int>(S.heads.size());
   S.f_s = static_cast<int>(S.chunks.size()) * c.ffn_chunk;
   S.hc = static_cast<int>(S.xheads.size());
+  S.pos_heads = positions_in(S.heads, U.heads);
+  S.pos_chunks = positions_in(S.chunks, U.chunks);
+  S.pos_xheads = positions_in(S.xheads, U.xheads);
   const int hd = S.h_s * dh, hcd = S.hc * dh, fs = S.f_s;
   const int N = P->N;
 
@@ -326,11 +385,27 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
   keep_alive.push_back(x_rows);
   keep_alive.push_back(x_segs);
 
+  // Union engine: the union rows of the step's FFN channels, which K1 gathers at every
+  // forward (the head-granular projections carry their maps in their kernel arguments).
+  if (uni) {
+    std::vector<int> up_rows;
+    for (int p : S.pos_chunks)
+      for (int j = 0; j < c.ffn_chunk; ++j) up_rows.push_back(p * c.ffn_chunk + j);
+    if ((e = upload_ints(P, up_rows, &S.up_rows_u, st)) || (e = upload_ints(P, S.pos_chunks, &S.down_segs_u, st)))
+      return e;
+    keep_alive.push_back(up_rows);
+  }
+
+  // per-step panels; under the union engine only the vectors (the weight matrices are read
+  // from the union through the maps) and, for the duration of plan creation, cWkv
   auto mk = [&](int which, long long rows, long long cols) -> dfs_status {
     Panel& p = S.P[which];
     p.rows = rows; p.cols = cols; p.ld = cols;
     if (rows * cols == 0) return DFS_OK;
-    return alloc_n(P, &p.p, rows * cols);
+    const bool matrix = which == 0 || which == 4 || which == 5 || which == 7 || which == 8 || which == 10 ||
+                        which == 14;
+    if (uni && matrix) return which == 10 ? alloc_temp(P, &p.p, rows * cols) : DFS_OK;
+    return alloc_weights(P, &p.p, rows * cols);
   };
   const bf16* wq = static_cast<const bf16*>(w.wq);
   const bf16* wk = static_cast<const bf16*>(w.wk);
@@ -345,27 +420,35 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
   }
   // K1 gathers
   if (hd > 0) {
-    bf16* Wqkv = S.P[0].p;
-    DFS_CK(dfs::launch_gather_rows(Wqkv, d, wq, d, d_qk_rows, hd, d, st));
-    DFS_CK(dfs::launch_gather_rows(Wqkv + static_cast<long long>(hd) * d, d, wk, d, d_qk_rows, hd, d, st));
-    DFS_CK(dfs::launch_gather_rows(Wqkv + 2LL * hd * d, d, wv, d, d_qk_rows, hd, d, st));
+    if (!uni) {
+      bf16* Wqkv = S.P[0].p;
+      DFS_CK(dfs::launch_gather_rows(Wqkv, d, wq, d, d_qk_rows, hd, d, st));
+      DFS_CK(dfs::launch_gather_rows(Wqkv + static_cast<long long>(hd) * d, d, wk, d, d_qk_rows, hd, d, st));
+      DFS_CK(dfs::launch_gather_rows(Wqkv + 2LL * hd * d, d, wv, d, d_qk_rows, hd, d, st));
+      DFS_CK(dfs::launch_gather_segs(S.P[4].p, hd, static_cast<const bf16*>(w.wo), d, d_qk_segs, hd / 8, d, st));
+    }
     bf16* b = S.P[1].p;
     DFS_CK(dfs::launch_gather_segs(b, 0, static_cast<const bf16*>(w.bq), 0, d_qk_segs, hd / 8, 1, st));
     DFS_CK(dfs::launch_gather_segs(b + hd, 0, static_cast<const bf16*>(w.bk), 0, d_qk_segs, hd / 8, 1, st));
     DFS_CK(dfs::launch_gather_segs(b + 2 * hd, 0, static_cast<const bf16*>(w.bv), 0, d_qk_segs, hd / 8, 1, st));
     DFS_CK(dfs::launch_gather_segs(S.P[2].p, 0, static_cast<const bf16*>(w.gq), 0, d_qk_segs, hd / 8, 1, st));
     DFS_CK(dfs::launch_gather_segs(S.P[3].p, 0, static_cast<const bf16*>(w.gk), 0, d_qk_segs, hd / 8, 1, st));
-    DFS_CK(dfs::launch_gather_segs(S.P[4].p, hd, static_cast<const bf16*>(w.wo), d, d_qk_segs, hd / 8, d, st));
   }
   if (fs > 0) {
     const int nch = static_cast<int>(S.chunks.size());
-    DFS_CK(dfs::launch_gather_rows(S.P[5].p, d, static_cast<const bf16*>(w.w_up), d, d_ffn_rows, fs, d, st));
+    if (!uni) {
+      DFS_CK(dfs::launch_gather_rows(S.P[5].p, d, static_cast<const bf16*>(w.w_up), d, d_ffn_rows, fs, d, st));
+      DFS_CK(dfs::launch_gather_segs(S.P[7].p, fs, static_cast<const bf16*>(w.w_down), c.ffn_dim, d_chunks, nch,
+                                     d, st));
+    }
     DFS_CK(dfs::launch_gather_segs(S.P[6].p, 0, static_cast<const bf16*>(w.b_up), 0, d_chunks, nch, 1, st));
-    DFS_CK(dfs::launch_gather_segs(S.P[7].p, fs, static_cast<const bf16*>(w.w_down), c.ffn_dim, d_chunks, nch, d,
-                                   st));
   }
   if (c.has_cross && hcd > 0) {
-    DFS_CK(dfs::launch_gather_rows(S.P[8].p, d, static_cast<const bf16*>(w.cwq), d, d_x_rows, hcd, d, st));
+    if (!uni) {
+      DFS_CK(dfs::launch_gather_rows(S.P[8].p, d, static_cast<const bf16*>(w.cwq), d, d_x_rows, hcd, d, st));
+      DFS_CK(dfs::launch_gather_segs(S.P[14].p, hcd, static_cast<const bf16*>(w.cwo), d, d_x_segs, hcd / 8, d,
+                                     st));
+    }
     DFS_CK(dfs::launch_gather_segs(S.P[9].p, 0, static_cast<const bf16*>(w.cbq), 0, d_x_segs, hcd / 8, 1, st));
     DFS_CK(dfs::launch_gather_rows(S.P[10].p, d, static_cast<const bf16*>(w.cwk), d, d_x_rows, hcd, d, st));
     DFS_CK(dfs::launch_gather_rows(S.P[10].p + static_cast<long long>(hcd) * d, d,
@@ -375,24 +458,52 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
                                    st));
     DFS_CK(dfs::launch_gather_segs(S.P[12].p, 0, static_cast<const bf16*>(w.cgq), 0, d_x_segs, hcd / 8, 1, st));
     DFS_CK(dfs::launch_gather_segs(S.P[13].p, 0, static_cast<const bf16*>(w.cgk), 0, d_x_segs, hcd / 8, 1, st));
-    DFS_CK(dfs::launch_gather_segs(S.P[14].p, hcd, static_cast<const bf16*>(w.cwo), d, d_x_segs, hcd / 8, d,
-                                   st));
   }
+
+  // Union engine: B of a head-granular projection read from the union panel through its
+  // map, in head units of the union.  Rows: group g (dh rows) of the step's [q | k | v] (or
+  // cross q) rows is head pos[g % h] of section g / h; padded to the B tiles of 256 rows.
+  // K columns: block k (64 columns) of the step's attention output is column block
+  // (pos[k dh_blocks] dh + ...) / 64 of the union.
+  const int nu = static_cast<int>(U.heads.size());
+  auto gather_rows = [&](dfs::GemmArgs& g, const std::vector<int>& pos, int sections, int nunion) -> dfs_status {
+    const int h = static_cast<int>(pos.size());
+    const size_t len = static_cast<size_t>((static_cast<long long>(sections) * h * dh + 255) / 256) * 256 / dh;
+    if (len > static_cast<size_t>(dfs::kGemmMapMax)) return fail(DFS_EUNSUPPORTED, "gather map too long");
+    g.b_gather = dfs::kGatherRows;
+    g.b_group = dh;
+    for (size_t i = 0; i < len; ++i) {
+      const int gi = static_cast<int>(std::min(i, static_cast<size_t>(sections * h - 1)));
+      g.b_idx[i] = static_cast<unsigned short>((gi / h) * nunion + pos[gi % h]);
+    }
+    return DFS_OK;
+  };
+  auto gather_kcols = [&](dfs::GemmArgs& g, const std::vector<int>& pos) -> dfs_status {
+    const int kb = static_cast<int>(pos.size()) * dh / 64;
+    if (kb > dfs::kGemmMapMax) return fail(DFS_EUNSUPPORTED, "gather map too long");
+    g.b_gather = dfs::kGatherKCols;
+    for (int k = 0; k < kb; ++k) g.b_idx[k] = static_cast<unsigned short>((pos[k * 64 / dh] * dh + (k * 64) % dh) / 64);
+    return DFS_OK;
+  };
 
   // kernel arguments
   const LayerConst& C = P->lc[l];
   CUtensorMap ma, mb;
   const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(dh)));
   if (hd > 0) {
-    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[0].p, d, 3LL * hd, d, 64, dfs::kGemmBRows))
-      return fail(DFS_ECUDA, "tensor map (QKV) failed");
+    const bool okb = uni ? make_map(&mb, U.wqkv.p, d, U.wqkv.rows, d, 64, dh)
+                         : make_map(&mb, S.P[0].p, d, 3LL * hd, d, 64, dfs::kGemmBRows);
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !okb) return fail(DFS_ECUDA, "tensor map (QKV) failed");
     S.g_qkv = gemm_args(P, ma, mb, N, 3 * hd, d, dfs::kEpiBias, S.P[1].p);
     S.g_qkv.out = P->qk; S.g_qkv.ldo = 2 * hd; S.g_qkv.split = 2 * hd;
     S.g_qkv.out_t = P->vt; S.g_qkv.ldt = P->vt_ld;
-    if (!make_map(&ma, P->attn, hd, N, hd, 64, 128) || !make_map(&mb, S.P[4].p, hd, d, hd, 64, dfs::kGemmBRows))
-      return fail(DFS_ECUDA, "tensor map (O) failed");
+    if (uni && (e = gather_rows(S.g_qkv, S.pos_heads, 3, nu))) return e;
+    const bool okbo = uni ? make_map(&mb, U.wo.p, U.wo.cols, d, U.wo.cols, 64, dfs::kGemmBRows)
+                          : make_map(&mb, S.P[4].p, hd, d, hd, 64, dfs::kGemmBRows);
+    if (!make_map(&ma, P->attn, hd, N, hd, 64, 128) || !okbo) return fail(DFS_ECUDA, "tensor map (O) failed");
     S.g_o = gemm_args(P, ma, mb, N, d, hd, dfs::kEpiGatedRes, C.bo);
     S.g_o.out = P->x1; S.g_o.ldo = d; S.g_o.out_f32 = 1; S.g_o.ldr = d; S.g_o.res_f32 = 0;
+    if (uni && (e = gather_kcols(S.g_o, S.pos_heads))) return e;
     dfs::AttnArgs& A = S.a_self;
     memset(&A, 0, sizeof(A));
     // a CTA pair of the attention kernel loads 64-key halves of K and DH/2-row halves of V^T
@@ -404,11 +515,14 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     A.out = P->attn; A.ldo = hd; A.scale_log2 = scale_log2; A.err = P->err;
   }
   if (fs > 0) {
-    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[5].p, d, fs, d, 64, dfs::kGemmBRows))
+    // union engine: the FFN panels live in the plan's per-forward scratch (same layout)
+    const bf16* wup = uni ? P->ffn_up_s : S.P[5].p;
+    const bf16* wdown = uni ? P->ffn_down_s : S.P[7].p;
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, wup, d, fs, d, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (up) failed");
     S.g_up = gemm_args(P, ma, mb, N, fs, d, dfs::kEpiBiasGelu, S.P[6].p);
     S.g_up.out = P->h; S.g_up.ldo = fs;
-    if (!make_map(&ma, P->h, fs, N, fs, 64, 128) || !make_map(&mb, S.P[7].p, fs, d, fs, 64, dfs::kGemmBRows))
+    if (!make_map(&ma, P->h, fs, N, fs, 64, 128) || !make_map(&mb, wdown, fs, d, fs, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (down) failed");
     S.g_down = gemm_args(P, ma, mb, N, d, fs, dfs::kEpiGatedRes, C.bdown);
     S.g_down.ldo = d; S.g_down.out_f32 = 0; S.g_down.res = P->x1; S.g_down.ldr = d; S.g_down.res_f32 = 1;
@@ -425,15 +539,19 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     DFS_CK(dfs::launch_gemm(kv, P->num_sms, st));
     DFS_CK(dfs::launch_qk_norm_rope(S.kc, hcd, c.ctx_len, 0, hcd, nullptr, S.P[13].p, dh, c.qk_norm_mode,
                                     c.ln_eps, nullptr, st));
-    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, S.P[8].p, d, hcd, d, 64, dfs::kGemmBRows))
-      return fail(DFS_ECUDA, "tensor map (cross q) failed");
+    const bool okq = uni ? make_map(&mb, U.cwq.p, d, U.cwq.rows, d, 64, dh)
+                         : make_map(&mb, S.P[8].p, d, hcd, d, 64, dfs::kGemmBRows);
+    if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !okq) return fail(DFS_ECUDA, "tensor map (cross q) failed");
     S.g_cq = gemm_args(P, ma, mb, N, hcd, d, dfs::kEpiBias, S.P[9].p);
     S.g_cq.out = P->qc; S.g_cq.ldo = hcd;
-    if (!make_map(&ma, P->attn, hcd, N, hcd, 64, 128) || !make_map(&mb, S.P[14].p, hcd, d, hcd, 64, dfs::kGemmBRows))
-      return fail(DFS_ECUDA, "tensor map (cross o) failed");
+    if (uni && (e = gather_rows(S.g_cq, S.pos_xheads, 1, static_cast<int>(U.xheads.size())))) return e;
+    const bool oko = uni ? make_map(&mb, U.cwo.p, U.cwo.cols, d, U.cwo.cols, 64, dfs::kGemmBRows)
+                         : make_map(&mb, S.P[14].p, hcd, d, hcd, 64, dfs::kGemmBRows);
+    if (!make_map(&ma, P->attn, hcd, N, hcd, 64, 128) || !oko) return fail(DFS_ECUDA, "tensor map (cross o) failed");
     S.g_co = gemm_args(P, ma, mb, N, d, hcd, dfs::kEpiGatedRes, C.cbo);
     S.g_co.out = P->x1; S.g_co.ldo = d; S.g_co.out_f32 = 1; S.g_co.res = P->x1; S.g_co.ldr = d;
     S.g_co.res_f32 = 1; S.g_co.gate = nullptr;
+    if (uni && (e = gather_kcols(S.g_co, S.pos_xheads))) return e;
     dfs::AttnArgs& A = S.a_cross;
     memset(&A, 0, sizeof(A));
     if (!make_map(&A.tma_q, P->qc, hcd, N, hcd, 64, 128) || !make_map(&A.tma_k, S.kc, hcd, c.ctx_len, hcd, 64, 64) ||
@@ -446,6 +564,82 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
   S.flops = 8 * Nd * dd * dh * S.h_s + 4 * Nd * Nd * dh * S.h_s + 4 * Nd * dd * S.f_s;
   if (c.has_cross)
     S.flops += 4 * Nd * dd * dh * S.hc + 4.0 * c.ctx_len * dd * dh * S.hc + 4 * Nd * c.ctx_len * dh * S.hc;
+  return DFS_OK;
+}
+
+// The layer's union super-model (Sec. 4.3): ids retained at any step (OR of the step gates;
+// block gates do not enter) and, under DFS_ENGINE_UNION, the weights of those units gathered
+// from the full layer once: Wqkv, Wo, W_up, W_down, cWq, cWo.
+dfs_status build_union(dfs_plan* P, int l, const dfs_layer_weights& w, const dfs_masks* m, cudaStream_t st,
+                       std::vector<std::vector<int>>& keep_alive) {
+  const dfs_config& c = P->cfg;
+  const int d = c.dim, H = c.n_heads, dh = c.head_dim, NC = c.ffn_dim / c.ffn_chunk;
+  LayerUnion& U = P->lu[l];
+  for (int h = 0; h < H; ++h) {
+    bool any = false, anyx = false;
+    for (int s = 0; s < P->T; ++s) {
+      const long long base = static_cast<long long>(s) * c.n_layers + l;
+      any |= m->head_gate[base * H + h] != 0;
+      anyx |= !m->xhead_gate || m->xhead_gate[base * H + h] != 0;
+    }
+    if (any) U.heads.push_back(h);
+    if (c.has_cross && anyx) U.xheads.push_back(h);
+  }
+  for (int k = 0; k < NC; ++k) {
+    bool any = false;
+    for (int s = 0; s < P->T; ++s) any |= m->ffn_gate[(static_cast<long long>(s) * c.n_layers + l) * NC + k] != 0;
+    if (any) U.chunks.push_back(k);
+  }
+  if (!P->uni) return DFS_OK;
+  const int nu = static_cast<int>(U.heads.size()), nf = static_cast<int>(U.chunks.size());
+  const int nx = static_cast<int>(U.xheads.size());
+  std::vector<int> rows, segs, frows, xrows, xsegs;
+  for (int h : U.heads)
+    for (int j = 0; j < dh; ++j) rows.push_back(h * dh + j);
+  for (int h : U.heads)
+    for (int j = 0; j < dh / 8; ++j) segs.push_back(h * dh / 8 + j);
+  for (int k : U.chunks)
+    for (int j = 0; j < c.ffn_chunk; ++j) frows.push_back(k * c.ffn_chunk + j);
+  for (int h : U.xheads)
+    for (int j = 0; j < dh; ++j) xrows.push_back(h * dh + j);
+  for (int h : U.xheads)
+    for (int j = 0; j < dh / 8; ++j) xsegs.push_back(h * dh / 8 + j);
+  int *d_rows, *d_segs, *d_frows, *d_chunks, *d_xrows, *d_xsegs;
+  dfs_status e;
+  if ((e = upload_ints(P, rows, &d_rows, st)) || (e = upload_ints(P, segs, &d_segs, st)) ||
+      (e = upload_ints(P, frows, &d_frows, st)) || (e = upload_ints(P, U.chunks, &d_chunks, st)) ||
+      (e = upload_ints(P, xrows, &d_xrows, st)) || (e = upload_ints(P, xsegs, &d_xsegs, st)))
+    return e;
+  for (auto* v : {&rows, &segs, &frows, &xrows, &xsegs}) keep_alive.push_back(*v);
+  auto mk = [&](Panel& p, long long r, long long cols) -> dfs_status {
+    p.rows = r; p.cols = cols; p.ld = cols;
+    return r * cols ? alloc_weights(P, &p.p, r * cols) : DFS_OK;
+  };
+  const long long ud = static_cast<long long>(nu) * dh, xd = static_cast<long long>(nx) * dh;
+  const long long uf = static_cast<long long>(nf) * c.ffn_chunk;
+  if ((e = mk(U.wqkv, 3 * ud, d)) || (e = mk(U.wo, d, ud)) || (e = mk(U.wup, uf, d)) || (e = mk(U.wdown, d, uf)))
+    return e;
+  if (c.has_cross && ((e = mk(U.cwq, xd, d)) || (e = mk(U.cwo, d, xd)))) return e;
+  if (ud > 0) {
+    const void* src[3] = {w.wq, w.wk, w.wv};
+    for (int q = 0; q < 3; ++q)
+      DFS_CK(dfs::launch_gather_rows(U.wqkv.p + q * ud * d, d, static_cast<const bf16*>(src[q]), d, d_rows,
+                                     static_cast<int>(ud), d, st));
+    DFS_CK(dfs::launch_gather_segs(U.wo.p, ud, static_cast<const bf16*>(w.wo), d, d_segs, static_cast<int>(ud / 8),
+                                   d, st));
+  }
+  if (uf > 0) {
+    DFS_CK(dfs::launch_gather_rows(U.wup.p, d, static_cast<const bf16*>(w.w_up), d, d_frows, static_cast<int>(uf),
+                                   d, st));
+    DFS_CK(dfs::launch_gather_segs(U.wdown.p, uf, static_cast<const bf16*>(w.w_down), c.ffn_dim, d_chunks, nf, d,
+                                   st));
+  }
+  if (c.has_cross && xd > 0) {
+    DFS_CK(dfs::launch_gather_rows(U.cwq.p, d, static_cast<const bf16*>(w.cwq), d, d_xrows, static_cast<int>(xd),
+                                   d, st));
+    DFS_CK(dfs::launch_gather_segs(U.cwo.p, xd, static_cast<const bf16*>(w.cwo), d, d_xsegs,
+                                   static_cast<int>(xd / 8), d, st));
+  }
   return DFS_OK;
 }
 
@@ -539,14 +733,25 @@ dfs_status create_impl(dfs_plan* P, const dfs_layer_weights* layers, const void*
       (e = alloc_n(P, &P->stage_out, N * d)) || (e = alloc_n(P, &P->stage_t, d)))
     return e;
   if (hmax > 0) DFS_CK(cudaMemsetAsync(P->vt, 0, sizeof(bf16) * hmax * dh * P->vt_ld, st));
+  if (P->uni && ((e = alloc_n(P, &P->ffn_up_s, static_cast<long long>(fmax) * d)) ||
+                 (e = alloc_n(P, &P->ffn_down_s, static_cast<long long>(fmax) * d))))
+    return e;
 
-  // per (step, layer): index tables, compacted panels, kernel arguments
+  // per layer: the union super-model; per (step, layer): index tables, compacted panels
+  // (or gather maps into the union), kernel arguments
   std::vector<std::vector<int>> keep_alive;  // host index lists stay valid until the sync below
+  P->lu.resize(P->L);
+  for (int l = 0; l < P->L; ++l)
+    if ((e = build_union(P, l, layers[l], m, st, keep_alive))) return e;
   P->sl.resize(static_cast<size_t>(P->T) * P->L);
   for (int s = 0; s < P->T; ++s)
     for (int l = 0; l < P->L; ++l)
       if ((e = build_step_layer(P, s, l, layers[l], m, ctx, st, keep_alive))) return e;
   DFS_CK(cudaStreamSynchronize(st));
+  // buffers needed only while the plan was built (union engine: the context K/V weights)
+  for (void* t : P->temps) cudaFree(t);
+  P->temps.clear();
+  for (StepLayer& S : P->sl) S.P[10].p = P->uni ? nullptr : S.P[10].p;
   int herr = 0;
   DFS_CK(cudaMemcpy(&herr, P->err, sizeof(int), cudaMemcpyDeviceToHost));
   if (herr) return fail(DFS_ETIMEOUT, "a kernel gave up waiting during plan creation");
@@ -554,6 +759,26 @@ dfs_status create_impl(dfs_plan* P, const dfs_layer_weights* layers, const void*
 }
 
 // ------------------------------------------------------------------ forward
+
+// Union engine: the step's FFN panels gathered from the layer's union (K1) into the plan's
+// scratch, read by the FFN projections right after (the paper's gather through I_t).
+// `profiled` = false launches without the per-kernel event bracket (the allocation-free
+// forward creates no events).
+dfs_status union_ffn_gather(dfs_plan* P, const StepLayer& S, int l, cudaStream_t st, bool profiled = true) {
+  if (!P->uni || S.f_s == 0) return DFS_OK;
+  const LayerUnion& U = P->lu[l];
+  const int d = P->cfg.dim, fs = S.f_s;
+  if (profiled) {
+    DFS_LAUNCH(DFS_K_GATHER, dfs::launch_gather_rows(P->ffn_up_s, d, U.wup.p, d, S.up_rows_u, fs, d, st));
+    DFS_LAUNCH(DFS_K_GATHER, dfs::launch_gather_segs(P->ffn_down_s, fs, U.wdown.p, U.wdown.ld, S.down_segs_u,
+                                                     fs / P->cfg.ffn_chunk, d, st));
+  } else {
+    DFS_CK(dfs::launch_gather_rows(P->ffn_up_s, d, U.wup.p, d, S.up_rows_u, fs, d, st));
+    DFS_CK(dfs::launch_gather_segs(P->ffn_down_s, fs, U.wdown.p, U.wdown.ld, S.down_segs_u, fs / P->cfg.ffn_chunk,
+                                   d, st));
+  }
+  return DFS_OK;
+}
 
 dfs_status forward_impl(dfs_plan* P, int s, int l, const bf16* x, bf16* out, cudaStream_t st) {
   // P->mod holds this layer's six modulation vectors
@@ -600,6 +825,8 @@ dfs_status forward_impl(dfs_plan* P, int s, int l, const bf16* x, bf16* out, cud
   }
   DFS_LAUNCH(DFS_K_ADALN, dfs::launch_row_norm(P->xm, P->x1, 1, N, d, scale_f, 1.f, shift_f, c.ln_eps, st));
   if (S.f_s > 0) {
+    dfs_status e = union_ffn_gather(P, S, l, st);
+    if (e) return e;
     DFS_LAUNCH(DFS_K_GEMM_UP, dfs::launch_gemm(S.g_up, P->num_sms, st));
     dfs::GemmArgs g = S.g_down;
     g.out = out;
@@ -645,6 +872,7 @@ dfs_status dfs_plan_create(const dfs_config* cfg, const dfs_layer_weights* layer
   dfs_plan* P = new (std::nothrow) dfs_plan();
   if (!P) return fail(DFS_ENOMEM, "host allocation failed");
   P->cfg = *cfg;
+  P->uni = cfg->engine == DFS_ENGINE_UNION;
   P->T = cfg->n_steps;
   P->L = cfg->n_layers;
   P->N = cfg->grid_t * cfg->grid_h * cfg->grid_w;
@@ -720,8 +948,12 @@ dfs_status dfs_plan_indices(const dfs_plan* P, int step, int layer, int kind, in
   if (!P || !count) return fail(DFS_EINVAL, "NULL plan or count");
   if (step < 0 || step >= P->T || layer < 0 || layer >= P->L) return fail(DFS_EINVAL, "step/layer out of range");
   const StepLayer& S = P->sl[step * P->L + layer];
-  const std::vector<int>* v = kind == 0 ? &S.heads : kind == 1 ? &S.chunks : kind == 2 ? &S.xheads : nullptr;
-  if (!v) return fail(DFS_EINVAL, "kind must be 0, 1 or 2");
+  const LayerUnion& U = P->lu[layer];
+  // kinds 0..2 the step's ids, 3..5 the union's ids, 6..8 the step's positions in the union
+  const std::vector<int>* lists[9] = {&S.heads,     &S.chunks,     &S.xheads,     &U.heads,     &U.chunks,
+                                      &U.xheads,    &S.pos_heads,  &S.pos_chunks, &S.pos_xheads};
+  if (kind < 0 || kind > 8) return fail(DFS_EINVAL, "kind must be in 0..8");
+  const std::vector<int>* v = lists[kind];
   *count = static_cast<int>(v->size());
   if (out)
     for (size_t i = 0; i < v->size(); ++i) out[i] = (*v)[i];
@@ -735,6 +967,26 @@ dfs_status dfs_plan_panel(const dfs_plan* P, int step, int layer, int which, con
   if (which < 0 || which > 14 || (which > 7 && !P->cfg.has_cross)) return fail(DFS_EINVAL, "bad panel id");
   const Panel& p = P->sl[step * P->L + layer].P[which];
   *dev = p.p; *rows = p.rows; *cols = p.cols; *ld = p.ld;
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_union_panel(const dfs_plan* P, int layer, int which, const void** dev, int64_t* rows,
+                                int64_t* cols, int64_t* ld) {
+  if (!P || !dev || !rows || !cols || !ld) return fail(DFS_EINVAL, "NULL argument");
+  if (layer < 0 || layer >= P->L) return fail(DFS_EINVAL, "layer out of range");
+  if (which < 0 || which > 5 || (which > 3 && !P->cfg.has_cross)) return fail(DFS_EINVAL, "bad union panel id");
+  if (!P->uni) return fail(DFS_EUNSUPPORTED, "the plan does not use DFS_ENGINE_UNION");
+  const LayerUnion& U = P->lu[layer];
+  const Panel* ps[6] = {&U.wqkv, &U.wo, &U.wup, &U.wdown, &U.cwq, &U.cwo};
+  const Panel& p = *ps[which];
+  *dev = p.p; *rows = p.rows; *cols = p.cols; *ld = p.ld;
+  return DFS_OK;
+}
+
+dfs_status dfs_plan_memory(const dfs_plan* P, int64_t* weight_bytes, int64_t* device_bytes) {
+  if (!P || !weight_bytes || !device_bytes) return fail(DFS_EINVAL, "NULL argument");
+  *weight_bytes = P->bytes_weights;
+  *device_bytes = P->bytes_total;
   return DFS_OK;
 }
 
@@ -961,6 +1213,9 @@ dfs_status noalloc_forward(dfs_plan* P, int s, int l, const bf16* x, const bf16*
   }
   DFS_CK(dfs::launch_row_norm(xm, x1, 1, N, d, mod + 4 * d, 1.f, mod + 3 * d, c.ln_eps, st));
   if (fs > 0) {
+    // union engine: FFN panels into the plan's scratch (allocated with the plan)
+    dfs_status eg = union_ffn_gather(P, S, l, st, false);
+    if (eg) return eg;
     dfs::GemmArgs u = S.g_up;
     if (!make_map(&u.tma_a, xm, d, N, d, 64, 128)) return fail(DFS_ECUDA, "tensor map (up) failed");
     u.out = h;

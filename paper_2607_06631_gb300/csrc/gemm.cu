@@ -8,7 +8,8 @@
 // B element from L2 once per tile.  Both CTAs' TMA loads complete on the even CTA's
 // barriers; its single MMA thread's commits are multicast to both CTAs.
 //
-//   warp 0      TMA producer: own A rows 128x64 and own B rows 128x64 per stage, 6-stage ring.
+//   warp 0      TMA producer: own A rows 128x64 and own B rows 128x64 per stage, 6-stage ring;
+//               B either as stored or gathered head by head from a union weight matrix.
 //   warp 1      TMEM allocation (collective over the pair); in the even CTA the MMA thread,
 //               issuing into one of two accumulators (2 x 256 fp32 columns per CTA), so the
 //               epilogue of tile i overlaps the main loop of tile i+1.
@@ -209,14 +210,34 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       for (int tile = pair; tile < num_tiles && !failed; tile += n_pairs) {
         int mt, nt;
         tile_coords(tile, m_tiles, n_tiles, p.group, mt, nt);
+        const int nb0 = nt * kGemmBN + static_cast<int>(rank) * kGemmBRows;  // this CTA's first B row
+        // kGatherRows: the union rows of this CTA's B half (one group of 128 rows, or two of
+        // 64) are the same for every K block.  A TMA instruction costs the issuing thread
+        // about 140 cycles (measured), so each stage issues exactly one B copy (two for
+        // 64-row groups), never a predicated run of them.
+        int row0 = 0, row1 = 0;
+        if (p.b_gather == kGatherRows) {
+          const int g0 = nb0 / p.b_group;
+          row0 = p.b_idx[g0] * p.b_group;
+          if (p.b_group == 64) row1 = p.b_idx[g0 + 1] * 64;
+        }
         for (int k = 0; k < kb; ++k) {
           if (!mbar_wait_cluster(&empty[stage], phase ^ 1, p.err)) { failed = true; break; }
           if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * kGemmStageBytes);
           const uint32_t lf = map_to_rank(&full[stage], 0);
           tma_load_2d_pair(sA + stage * kGemmABytes, &p.tma_a, lf, k * kGemmBK,
                            mt * kGemmTileM + static_cast<int>(rank) * kGemmBM);
-          tma_load_2d_pair(sB + stage * kGemmBBytes, &p.tma_b, lf, k * kGemmBK,
-                           nt * kGemmBN + static_cast<int>(rank) * kGemmBRows);
+          uint8_t* dB = sB + stage * kGemmBBytes;
+          if (p.b_gather == kGatherNone) {
+            tma_load_2d_pair(dB, &p.tma_b, lf, k * kGemmBK, nb0);
+          } else if (p.b_gather == kGatherRows) {
+            // 64-row groups stack in the same 128-byte swizzled layout one 128-row box
+            // produces (8-row atoms of 1024 B)
+            tma_load_2d_pair(dB, &p.tma_b, lf, k * kGemmBK, row0);
+            if (p.b_group == 64) tma_load_2d_pair(dB + 64 * 128, &p.tma_b, lf, k * kGemmBK, row1);
+          } else {  // kGatherKCols
+            tma_load_2d_pair(dB, &p.tma_b, lf, p.b_idx[k] * kGemmBK, nb0);
+          }
           if (++stage == kGemmStages) { stage = 0; phase ^= 1; }
         }
       }

@@ -24,9 +24,25 @@ constexpr int kGemmBBytes = kGemmBRows * kGemmBK * 2;
 constexpr int kGemmStageBytes = kGemmABytes + kGemmBBytes;
 constexpr int kGemmSmem = kGemmStages * kGemmStageBytes + 1024 + 256;
 
+// How the B operand reaches shared memory.  kGatherNone reads B [N, K] as stored; the other
+// modes read a union weight matrix (the parameters retained at any step, Sec. 4.3) through
+// a per-step index map, one whole attention head at a time, so that the step's weights never
+// exist as a separate copy:
+//   kGatherRows    B rows (output features) in groups of b_group = head_dim rows (64 or 128):
+//                  group g of the step is union row b_idx[g] * b_group of [N_union, K].
+//   kGatherKCols   K block k (64 columns) of the step is union column b_idx[k] * 64 of
+//                  [N, K_union] (head_dim a multiple of 64, so K has no tail).
+// The map travels in the kernel parameters: indexed by tile / K-block counters it is read
+// with uniform constant loads, so the TMA coordinates need no per-copy conversion from a
+// per-thread register.  kGatherRows maps are padded (repeating the last entry) to
+// n_tiles * 256 / b_group entries, so that every group a CTA stages, including groups past
+// N, reads a valid row; those rows land in output columns that are never stored.
+enum GatherMode : int { kGatherNone = 0, kGatherRows = 1, kGatherKCols = 2 };
+constexpr int kGemmMapMax = 512;  // entries: 3 * 8192 / 64 row groups, 8192 / 64 K blocks
+
 struct GemmArgs {
   CUtensorMap tma_a;  // A [M, K], box {64, 128}, 128 B swizzle
-  CUtensorMap tma_b;  // B [N, K], box {64, 128}, 128 B swizzle
+  CUtensorMap tma_b;  // B [N, K], box {64, 128}, 128 B swizzle (see GatherMode for the others)
   int M, N, K;
   int mode;
   const bf16* bias;  // [N] or null
@@ -41,6 +57,9 @@ struct GemmArgs {
   int res_f32;
   const float* gate;  // [N] or null (gate = 1)
   int group;          // M tiles per raster group (tiles of one group sweep N together)
+  int b_gather;       // GatherMode
+  int b_group;        // kGatherRows: rows per group (64 or 128)
+  unsigned short b_idx[kGemmMapMax];  // index map of the gather (see GatherMode)
   int* err;
 };
 

@@ -22,16 +22,23 @@ _STATUS = {0: "DFS_OK", 1: "DFS_EINVAL", 2: "DFS_ENOMEM", 3: "DFS_ECUDA", 4: "DF
 
 EXPORTED = ("dfs_plan_create", "dfs_block_forward", "dfs_block_forward_layer", "dfs_block_forward_host",
             "dfs_block_forward_noalloc",
-            "dfs_denoise", "dfs_plan_indices", "dfs_plan_panel", "dfs_plan_flops", "dfs_plan_workspace",
+            "dfs_denoise", "dfs_plan_indices", "dfs_plan_panel", "dfs_plan_union_panel", "dfs_plan_memory",
+            "dfs_plan_flops", "dfs_plan_workspace",
             "dfs_plan_sync", "dfs_selftest_wait_timeout", "dfs_plan_profile", "dfs_plan_profile_read", "dfs_gates_from_soft_masks",
             "dfs_plan_destroy", "dfs_last_error")
 
 KERNEL_KINDS = ("modulation", "adaln", "gemm_qkv", "qk_norm_rope", "attention", "gemm_o", "gemm_up",
-                "gemm_down", "cross", "other")
+                "gemm_down", "cross", "other", "gather")
 
 PANELS = {"wqkv": 0, "bqkv": 1, "gq": 2, "gk": 3, "wo": 4, "w_up": 5, "b_up": 6, "w_down": 7,
           "cwq": 8, "cbq": 9, "cwkv": 10, "cbkv": 11, "cgq": 12, "cgk": 13, "cwo": 14}
 WORKSPACE = {"xm": 0, "qk": 1, "vt": 2, "attn": 3, "x1": 4, "h": 5, "mod": 6}
+UNION_PANELS = {"wqkv": 0, "wo": 1, "w_up": 2, "w_down": 3, "cwq": 4, "cwo": 5}
+DFS_ENGINE_COMPACTED, DFS_ENGINE_UNION = 0, 1
+ENGINES = {"compacted": DFS_ENGINE_COMPACTED, "union": DFS_ENGINE_UNION}
+# dfs_plan_indices kinds
+INDEX_KINDS = {"heads": 0, "chunks": 1, "xheads": 2, "union_heads": 3, "union_chunks": 4, "union_xheads": 5,
+               "pos_heads": 6, "pos_chunks": 7, "pos_xheads": 8}
 
 
 class DfsError(RuntimeError):
@@ -43,7 +50,8 @@ class DfsError(RuntimeError):
 class dfs_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in ("dim", "n_heads", "head_dim", "ffn_dim", "ffn_chunk", "n_layers",
                                             "n_steps", "grid_t", "grid_h", "grid_w", "ctx_len", "has_cross")] + \
-               [("ln_eps", ctypes.c_float), ("rope_theta", ctypes.c_float), ("qk_norm_mode", ctypes.c_int)]
+               [("ln_eps", ctypes.c_float), ("rope_theta", ctypes.c_float), ("qk_norm_mode", ctypes.c_int),
+                ("engine", ctypes.c_int)]
 
 
 LAYER_FIELDS = ("wq", "bq", "wk", "bk", "wv", "bv", "wo", "bo", "gq", "gk", "w_up", "b_up", "w_down", "b_down",
@@ -79,6 +87,8 @@ def lib() -> ctypes.CDLL:
         L.dfs_denoise.argtypes = [vp, vp, i32, vp, vp]
         L.dfs_plan_indices.argtypes = [vp, i32, i32, i32, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(i32)]
         L.dfs_plan_panel.argtypes = [vp, i32, i32, i32, ctypes.POINTER(vp), i64p, i64p, i64p]
+        L.dfs_plan_union_panel.argtypes = [vp, i32, i32, ctypes.POINTER(vp), i64p, i64p, i64p]
+        L.dfs_plan_memory.argtypes = [vp, i64p, i64p]
         L.dfs_plan_flops.argtypes = [vp, i32, i32, ctypes.POINTER(ctypes.c_double)]
         L.dfs_plan_workspace.argtypes = [vp, i32, ctypes.POINTER(vp), i64p, i64p, i64p, ctypes.POINTER(i32)]
         L.dfs_plan_sync.argtypes = [vp, vp]
@@ -141,6 +151,11 @@ def make_config(cfg: Any) -> dfs_config:
     c.grid_t, c.grid_h, c.grid_w = int(grid[0]), int(grid[1]), int(grid[2])
     c.ctx_len, c.has_cross = g("ctx_len"), g("has_cross")
     c.ln_eps, c.rope_theta, c.qk_norm_mode = g("ln_eps"), g("rope_theta"), g("qk_norm_mode")
+    try:
+        eng = g("engine")
+    except (KeyError, AttributeError):
+        eng = DFS_ENGINE_COMPACTED
+    c.engine = ENGINES[eng] if isinstance(eng, str) else int(eng)
     return c
 
 
@@ -220,7 +235,9 @@ def dfs_denoise(plan, latents, n_steps: int, t_embs, stream=None):
     _check(lib().dfs_denoise(_h(plan), _ptr(latents), n_steps, _ptr(t_embs), _stream(stream)))
 
 
-def dfs_plan_indices(plan, step: int, layer: int, kind: int) -> np.ndarray:
+def dfs_plan_indices(plan, step: int, layer: int, kind) -> np.ndarray:
+    """Index list of (step, layer); `kind` is an int or a name of INDEX_KINDS."""
+    kind = INDEX_KINDS[kind] if isinstance(kind, str) else kind
     n = ctypes.c_int()
     _check(lib().dfs_plan_indices(_h(plan), step, layer, kind, None, ctypes.byref(n)))
     out = np.zeros(n.value, dtype=np.int32)
@@ -236,6 +253,22 @@ def dfs_plan_panel(plan, step: int, layer: int, which):
     _check(lib().dfs_plan_panel(_h(plan), step, layer, w, ctypes.byref(p), ctypes.byref(r), ctypes.byref(c),
                                 ctypes.byref(ld)))
     return p.value or 0, r.value, c.value, ld.value
+
+
+def dfs_plan_union_panel(plan, layer: int, which):
+    """(device address, rows, cols, ld) of a union panel (DFS_ENGINE_UNION plans)."""
+    w = UNION_PANELS[which] if isinstance(which, str) else which
+    p, r, c, ld = ctypes.c_void_p(), ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+    _check(lib().dfs_plan_union_panel(_h(plan), layer, w, ctypes.byref(p), ctypes.byref(r), ctypes.byref(c),
+                                      ctypes.byref(ld)))
+    return p.value or 0, r.value, c.value, ld.value
+
+
+def dfs_plan_memory(plan):
+    """(weight bytes, device bytes) held by the plan."""
+    wb, db = ctypes.c_int64(), ctypes.c_int64()
+    _check(lib().dfs_plan_memory(_h(plan), ctypes.byref(wb), ctypes.byref(db)))
+    return wb.value, db.value
 
 
 def dfs_plan_flops(plan, step: int, layer: int = 0) -> float:

@@ -51,6 +51,14 @@ def read_panel(plan, step: int, layer: int, which) -> np.ndarray:
     return to_bits(view_device(p, r, c, ld, 0).clone())
 
 
+def read_union_panel(plan, layer: int, which) -> np.ndarray:
+    """Union panel (DFS_ENGINE_UNION) as uint16 bf16 bits [rows, cols] (host copy)."""
+    p, r, c, ld = dfs.dfs_plan_union_panel(plan, layer, which)
+    if r * c == 0:
+        return np.zeros((r, c), np.uint16)
+    return to_bits(view_device(p, r, c, ld, 0).clone())
+
+
 def read_workspace(plan, which) -> np.ndarray:
     """Workspace buffer of the last forward: float64 array [rows, cols]."""
     p, r, c, ld, dt = dfs.dfs_plan_workspace(plan, which)

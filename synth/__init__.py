@@ -74,6 +74,7 @@ class Config:
     rope_theta: float = 10000.0
     qk_norm_mode: int = 0
     block_gate: Optional[List[List[int]]] = None  # [n_steps][n_layers]; None -> all ones
+    engine: int = 0        # how the library holds the weights: 0 per-step copies, 1 union
 
     @property
     def n_tokens(self) -> int:

@@ -72,3 +72,34 @@ def test_720p_block_half_keep():
     errs = run_large(cfg, (5,), edge=32, spread=64)  # step 5 keeps 20 heads / 6912 channels
     for s, (e, b) in errs.items():
         assert e <= TOL and b <= TOL, (s, e, b)
+
+
+def test_wan14b_union_engine_bit_identical_to_compacted():
+    """The union engine (one union super-model, TMA gathers through I_t) gives the
+    compacted engine's output bit for bit at full size, with less weight memory."""
+    import copy
+    import torch
+    from paper_2607_06631_gb300 import build, dfs, host
+    build.build()
+    cfg = synth.wan14b()
+    shared, layers, masks, acts = synth.make_problem(cfg)
+    outs, mem = {}, {}
+    for eng in (0, 1):
+        c = copy.deepcopy(cfg)
+        c.engine = eng
+        prob = host.DeviceProblem(c, shared, layers, masks, acts)
+        prob.create_plan()
+        prob.free_weights()
+        mem[eng] = dfs.dfs_plan_memory(prob.plan)[0]
+        out = torch.empty_like(prob.x)
+        for s in (0, 1, 3):
+            dfs.dfs_block_forward(prob.plan, s, prob.x, prob.t_emb[s], out)
+            dfs.dfs_plan_sync(prob.plan)
+            outs[(eng, s)] = host.to_bits(out)
+        del prob
+        torch.cuda.empty_cache()
+    for s in (0, 1, 3):
+        np.testing.assert_array_equal(outs[(1, s)], outs[(0, s)], err_msg="step %d" % s)
+    # step 0 keeps every unit, so the union is the full layer (4 d^2 + 2 d F bf16 = 493 MB);
+    # the compacted engine holds the four steps' copies (1503 MB)
+    assert 0.49e9 < mem[1] < 0.50e9 and 1.50e9 < mem[0] < 1.51e9

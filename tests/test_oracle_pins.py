@@ -74,6 +74,72 @@ def test_compact_panels_are_row_and_column_selections():
     np.testing.assert_array_equal(P["w_down"][:, 8:16], lw["w_down"][:, c0 * 8:(c0 + 1) * 8])
 
 
+# --------------------------------------------------------------------------- union super-model (Sec. 4.3)
+
+def _hand_masks():
+    """Tiny config, one layer, hand-made gates: head 1 and chunk 5 are kept at no step."""
+    cfg = synth.tiny(has_cross=1)
+    m = synth.make_masks(cfg)
+    m["head_gate"][:, 0, :] = np.array([[1, 0, 0, 1], [0, 0, 1, 1], [0, 0, 0, 1], [1, 0, 0, 0]])
+    m["xhead_gate"][:, 0, :] = np.array([[0, 0, 0, 1], [0, 0, 0, 1], [0, 1, 0, 0], [0, 1, 0, 1]])
+    m["ffn_gate"][:] = 0
+    m["ffn_gate"][0, 0, [0, 7]] = 1
+    m["ffn_gate"][1, 0, [3]] = 1
+    m["ffn_gate"][3, 0, [3, 7, 9]] = 1
+    return cfg, m
+
+
+def test_union_tables_on_hand_made_gates():
+    cfg, m = _hand_masks()
+    u = O.union_tables(cfg, m, 0)
+    assert u["heads"].tolist() == [0, 2, 3]
+    assert [p.tolist() for p in u["pos_heads"]] == [[0, 2], [1, 2], [2], [0]]
+    assert u["chunks"].tolist() == [0, 3, 7, 9]
+    assert [p.tolist() for p in u["pos_chunks"]] == [[0, 2], [1], [], [1, 2, 3]]
+    assert u["xheads"].tolist() == [1, 3]
+    assert [p.tolist() for p in u["pos_xheads"]] == [[1], [1], [0], [0, 1]]
+
+
+def test_union_with_a_keep_all_step_is_every_unit():
+    cfg = synth.tiny()          # step 0 keeps all 4 heads and all 128 chunks
+    u = O.union_tables(cfg, synth.make_masks(cfg), 0)
+    assert u["heads"].tolist() == list(range(cfg.n_heads))
+    assert u["chunks"].tolist() == list(range(cfg.n_chunks))
+    assert u["pos_heads"][0].tolist() == list(range(cfg.n_heads))
+
+
+@pytest.mark.parametrize("hand", [False, True])
+def test_union_panels_indexed_by_positions_are_the_step_panels(hand):
+    """theta_union gathered through I_t gives exactly the exported per-step weights."""
+    if hand:
+        cfg, m = _hand_masks()
+    else:
+        cfg = synth.tiny(has_cross=1)
+        cfg.heads_kept = [[2], [3], [1], [2]]
+        cfg.chunks_kept = [[40], [90], [7], [64]]
+        m = synth.make_masks(cfg, "union")
+    lw = synth.make_layer(cfg, 0)
+    u = O.union_tables(cfg, m, 0)
+    U = O.union_panels(cfg, lw, u)
+    dh, C = cfg.head_dim, cfg.ffn_chunk
+    nu = len(u["heads"])
+    for s in range(cfg.n_steps):
+        P = O.compact_panels(lw, O.compact_indices(cfg, m, s, 0))
+        ph = np.asarray(u["pos_heads"][s], dtype=np.int64)
+        r = (ph[:, None] * dh + np.arange(dh)[None, :]).reshape(-1)
+        rows = np.concatenate([r, nu * dh + r, 2 * nu * dh + r])
+        np.testing.assert_array_equal(U["wqkv"][rows], P["wqkv"])
+        np.testing.assert_array_equal(U["wo"][:, r], P["wo"])
+        pc = np.asarray(u["pos_chunks"][s], dtype=np.int64)
+        ch = (pc[:, None] * C + np.arange(C)[None, :]).reshape(-1)
+        np.testing.assert_array_equal(U["w_up"][ch], P["w_up"])
+        np.testing.assert_array_equal(U["w_down"][:, ch], P["w_down"])
+        px = np.asarray(u["pos_xheads"][s], dtype=np.int64)
+        xr = (px[:, None] * dh + np.arange(dh)[None, :]).reshape(-1)
+        np.testing.assert_array_equal(U["cwq"][xr], P["cwq"])
+        np.testing.assert_array_equal(U["cwo"][:, xr], P["cwo"])
+
+
 # --------------------------------------------------------------------------- elementary ops
 
 def test_linear_orientation_out_in():
