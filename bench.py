@@ -17,6 +17,7 @@ sample.  `--impl reference` times that CPU oracle alone (the reference arm).
 from __future__ import annotations
 
 import argparse
+import copy
 import json
 import os
 import statistics
@@ -67,14 +68,26 @@ def _named_config(name: str):
         return synth.wan13b()
     if name == "tiny":
         return synth.tiny()
+    if name == "wan13b_policy":
+        return synth.wan13b_policy()
     if name.startswith("sweep720:"):
         return synth.sweep720(float(name.split(":")[1]))
     raise SystemExit("unknown config " + name)
 
 
+def _policy_shaped(cfg) -> bool:
+    return any(len(set(h)) > 1 for h in cfg.heads_kept) or any(len(set(c)) > 1 for c in cfg.chunks_kept)
+
+
 def workload_desc(cfg) -> str:
-    hk = "/".join(str(cfg.heads_kept[s][0]) for s in range(cfg.n_steps))
-    fk = "/".join(str(8 * cfg.chunks_kept[s][0]) for s in range(cfg.n_steps))
+    if _policy_shaped(cfg):
+        hk = "/".join("%d-%d" % (min(cfg.heads_kept[s]), max(cfg.heads_kept[s])) for s in range(cfg.n_steps))
+        fk = "/".join("%d-%d" % (8 * min(cfg.chunks_kept[s]), 8 * max(cfg.chunks_kept[s]))
+                      for s in range(cfg.n_steps))
+        hk += " per layer (policy-shaped: U-shaped per-step retention, deep layers pruned most)"
+    else:
+        hk = "/".join(str(cfg.heads_kept[s][0]) for s in range(cfg.n_steps))
+        fk = "/".join(str(8 * cfg.chunks_kept[s][0]) for s in range(cfg.n_steps))
     what = ("%d-layer %d-step denoise (dfs_denoise)" % (cfg.n_layers, cfg.n_steps) if cfg.n_layers > 1
             else "%d MoM steps per bench step" % cfg.n_steps)
     cross = (", text cross-attention over %d context tokens (cross heads kept as self heads)" % cfg.ctx_len
@@ -88,8 +101,8 @@ def workload_desc(cfg) -> str:
 def panel_mb(cfg):
     """Smallest and largest per-step compacted weight bytes of one layer (MB)."""
     d, dh = cfg.dim, cfg.head_dim
-    mb = [(4 * cfg.heads_kept[s][0] * dh * d + 2 * 8 * cfg.chunks_kept[s][0] * d) * 2 / 1e6
-          for s in range(cfg.n_steps)]
+    mb = [(4 * cfg.heads_kept[s][l] * dh * d + 2 * 8 * cfg.chunks_kept[s][l] * d) * 2 / 1e6
+          for s in range(cfg.n_steps) for l in range(cfg.n_layers)]
     return min(mb), max(mb)
 
 
@@ -99,22 +112,22 @@ def kernel_units(cfg):
     N, d, dh = cfg.n_tokens, cfg.dim, cfg.head_dim
     u = {k: 0.0 for k in KINDS}
     for s in range(cfg.n_steps):
-        hd = cfg.heads_kept[s][0] * dh
-        fs = 8 * cfg.chunks_kept[s][0]
-        u["gemm_qkv"] += 2.0 * N * d * 3 * hd
-        u["attention"] += 4.0 * N * N * hd
-        u["gemm_o"] += 2.0 * N * hd * d
-        u["gemm_up"] += 2.0 * N * d * fs
-        u["gemm_down"] += 2.0 * N * fs * d
-        u["adaln"] += N * d * (2 + 2) + N * d * (4 + 2)      # x bf16 -> xm, x1 fp32 -> xm2
-        u["qk_norm_rope"] += 2.0 * N * 2 * hd * 2              # q, k read + written
-        u["modulation"] += 6.0 * d * d * 2                     # W_t read once
-        if cfg.engine == 1:                                    # union engine: FFN panels gathered
-            u["gather"] += 2.0 * (2 * fs * d * 2)              # W_up_s, W_down_s read + written
-        if cfg.has_cross:
-            hc = cfg.xheads_kept[s][0] * dh
-            u["cross"] += 4.0 * N * d * hc + 4.0 * N * cfg.ctx_len * hc
-    u = {k: v * cfg.n_layers for k, v in u.items()}
+        for l in range(cfg.n_layers):
+            hd = cfg.heads_kept[s][l] * dh
+            fs = 8 * cfg.chunks_kept[s][l]
+            u["gemm_qkv"] += 2.0 * N * d * 3 * hd
+            u["attention"] += 4.0 * N * N * hd
+            u["gemm_o"] += 2.0 * N * hd * d
+            u["gemm_up"] += 2.0 * N * d * fs
+            u["gemm_down"] += 2.0 * N * fs * d
+            u["adaln"] += N * d * (2 + 2) + N * d * (4 + 2)      # x bf16 -> xm, x1 fp32 -> xm2
+            u["qk_norm_rope"] += 2.0 * N * 2 * hd * 2              # q, k read + written
+            u["modulation"] += 6.0 * d * d * 2                     # W_t read once
+            if cfg.engine == 1:                                    # union engine: FFN panels gathered
+                u["gather"] += 2.0 * (2 * fs * d * 2)              # W_up_s, W_down_s read + written
+            if cfg.has_cross:
+                hc = cfg.xheads_kept[s][l] * dh
+                u["cross"] += 4.0 * N * d * hc + 4.0 * N * cfg.ctx_len * hc
     if cfg.n_layers > 1:  # the stack's modulation GEMV runs once per step, not per layer
         u["modulation"] = cfg.n_steps * 6.0 * d * d * 2
     bound = {k: ("tensor" if k.startswith("gemm") or k in ("attention", "cross") else "hbm") for k in KINDS}
@@ -316,16 +329,35 @@ def run_ours(args):
     cfg.engine = dfs.ENGINES[args.engine]
     T, L = cfg.n_steps, cfg.n_layers
     stream = torch.cuda.current_stream()
+    # the dense reference of the speedups: step 0 when it keeps every unit, else a separate
+    # one-step plan over the same weights that keeps every unit
+    dense_step0 = all(h == cfg.n_heads for h in cfg.heads_kept[0]) and \
+        all(c == cfg.n_chunks for c in cfg.chunks_kept[0]) and \
+        (not cfg.has_cross or all(h == cfg.n_heads for h in cfg.xheads_kept[0]))
+    dense_plan = None
+
+    def make_dense(layers_dev, w_t_dev, b_t_dev, ctx_dev):
+        dc = copy.deepcopy(cfg)
+        dc.n_steps = 1
+        ones = {"block_gate": np.ones((1, L), np.uint8), "head_gate": np.ones((1, L, cfg.n_heads), np.uint8),
+                "xhead_gate": np.ones((1, L, cfg.n_heads), np.uint8) if cfg.has_cross else None,
+                "ffn_gate": np.ones((1, L, cfg.n_chunks), np.uint8)}
+        return dfs.dfs_plan_create(dc, layers_dev, w_t_dev, b_t_dev, ones, ctx_dev, stream)
+
     if L == 1:
         shared, layers, masks, acts = synth.make_problem(cfg)
         prob = host.DeviceProblem(cfg, shared, layers, masks, acts)
         del shared, layers
         plan = prob.create_plan(stream)
+        if not dense_step0:
+            dense_plan = make_dense(prob.layers, prob.w_t, prob.b_t, prob.ctx)
         prob.free_weights()
         x, temb = prob.x, prob.t_emb
     else:
         dl, w_t, b_t, masks, x, temb, ctx = device_stack(cfg)
         plan = dfs.dfs_plan_create(cfg, dl, w_t, b_t, masks, ctx, stream)
+        if not dense_step0:
+            dense_plan = make_dense(dl, w_t, b_t, ctx)
         del dl, w_t, b_t
         torch.cuda.empty_cache()
         prob = None
@@ -405,25 +437,41 @@ def run_ours(args):
                                             else "hbm_gbs")}
 
     # per-MoM-step latency: pruned vs dense (step 0 keeps every head and channel)
-    step_ms = []
-    reps = max(3, min(10, args.steps)) if L == 1 else 0
-    for s in (range(T) if L == 1 else ()):
-        for _ in range(2):
-            dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
+    # per-MoM-step latency (every layer of the step, as the denoising loop runs it) against the
+    # dense reference
+    bufs = (out, torch.empty_like(x)) if L > 1 else (out,)
+
+    def run_step(pl, s):
+        cur = x
+        for l in range(L):
+            dst = bufs[l % len(bufs)]
+            dfs.dfs_block_forward_layer(pl, s, l, cur, temb[s], dst, stream)
+            cur = dst
+
+    def time_step(pl, s):
+        reps = max(3, min(10, args.steps)) if L == 1 else 2
+        for _ in range(2 if L == 1 else 1):
+            run_step(pl, s)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         for _ in range(reps):
-            dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
+            run_step(pl, s)
         b.record(stream)
         torch.cuda.synchronize()
-        step_ms.append(a.elapsed_time(b) / reps)
-    ideal = [flops[0] / f for f in flops]
-    mean_ideal = flops[0] / (sum(flops) / T)
-    if step_ms:
-        speed = [step_ms[0] / t for t in step_ms]
-        mean_meas = step_ms[0] / (sum(step_ms) / T)
-    else:  # the stack runs its steps inside dfs_denoise; per-step speedups are not separated
-        speed, mean_meas = None, None
+        return a.elapsed_time(b) / reps
+
+    step_ms = [time_step(plan, s) for s in range(T)]
+    if dense_plan is None:
+        ref_ms, ref_flops, ref_desc = step_ms[0], flops[0], "step 0 (keeps every unit)"
+    else:
+        ref_ms = time_step(dense_plan, 0)
+        ref_flops = sum(dfs.dfs_plan_flops(dense_plan, 0, l) for l in range(L))
+        ref_desc = "separate plan keeping every unit (%.2f ms)" % ref_ms
+        dense_plan.close()
+    ideal = [ref_flops / f for f in flops]
+    mean_ideal = ref_flops / (sum(flops) / T)
+    speed = [ref_ms / t for t in step_ms]
+    mean_meas = ref_ms / (sum(step_ms) / T)
 
     # end to end through the host-buffer entry point (pinned host memory)
     e2e = None
@@ -468,6 +516,7 @@ def run_ours(args):
             "peak_tflops": peaks["bf16_tflops_sustained"], "peak_source": peak_src + " bf16_tflops_sustained",
             "step_ms": [round(t, 4) for t in step_ms], "step_tflops": [round(f / t / 1e9, 1) for f, t in
                                                                        zip(flops, step_ms)],
+            "step_flop_keep": [round(f / ref_flops, 4) for f in flops], "speedup_reference": ref_desc,
             "speedup": [round(v, 4) for v in speed] if speed else None,
             "speedup_ideal": [round(v, 4) for v in ideal],
             "speedup_vs_ideal": [round(a / b, 4) for a, b in zip(speed, ideal)] if speed else None,
@@ -492,7 +541,8 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--config", default="wan14b",
                     help="wan14b (default), wan13b, wan14b_cross, sweep720 (keep 1.0..0.5 as six steps), "
-                         "sweep720:<ratio>, wan14b_x<L> (L-layer 4-step denoise with cross-attention), tiny")
+                         "sweep720:<ratio>, wan14b_x<L> (L-layer 4-step denoise with cross-attention), "
+                         "wan13b_policy (30-layer 4-step denoise, policy-shaped masks), tiny")
     ap.add_argument("--grid", default=None, help="override the latent grid T,H,W (smaller profiling cases)")
     ap.add_argument("--engine", choices=("compacted", "union"), default="compacted",
                     help="weights per (step, layer) compacted once (default), or one union super-model per "

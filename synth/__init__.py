@@ -154,6 +154,57 @@ def wan14b_cross() -> Config:
                          (1.0, 0.8, 0.7, 0.55), has_cross=1, ctx_len=512)
 
 
+# Per-step keep profiles shaped like the learned pruning policy the paper analyses (Sec. 6,
+# "U-shaped computational allocation" and "semantic freezing in deep layers"; App. D): the two
+# end steps keep more than the two middle ones, deeper layers lose more self / cross-attention
+# heads than shallow ones (most at t2 and t3, where the deepest layer is shut down), and the FFN
+# keeps more than attention.  At depth u = l / (L - 1) of step s, a unit kind keeps
+#     clip(k0 - slope * u, 0, 1)
+# of its heads (self and cross alike) / FFN chunks, per step
+#     (attention k0, attention slope, FFN k0, FFN slope).
+# The constants were chosen so that the 30-layer Wan-1.3B-shaped stack with cross-attention at
+# 32760 tokens keeps 88.6 / 78.7 / 77.1 / 89.1 % of its dense FLOPs per step (the paper's learned
+# policy: 88.4 / 78.5 / 77.1 / 89.1 %; mean 83.3 % against the final checkpoint's ~83 %).
+POLICY_PROFILE = ((1.095, 0.40, 0.97, 0.12),
+                  (2.307, 2.30, 0.90, 0.20),
+                  (2.282, 2.30, 0.90, 0.20),
+                  (1.096, 0.40, 0.97, 0.12))
+
+
+def policy_counts(n_heads: int, n_chunks: int, n_layers: int, profile=POLICY_PROFILE):
+    """[n_steps][n_layers] retained head and FFN chunk counts of the policy-shaped profile."""
+    heads, chunks = [], []
+    for a0, ba, f0, bf in profile:
+        hs, cs = [], []
+        for l in range(n_layers):
+            u = l / (n_layers - 1) if n_layers > 1 else 0.0
+            a = min(1.0, max(0.0, a0 - ba * u))
+            f = min(1.0, max(0.0, f0 - bf * u))
+            hs.append(keep_count(a, n_heads))
+            cs.append(keep_count(f, n_chunks))
+        heads.append(hs)
+        chunks.append(cs)
+    return heads, chunks
+
+
+def wan13b_policy(n_layers: int = 30, grid=(21, 30, 52)) -> Config:
+    """Wan-1.3B-shaped stack (30 blocks, d=1536, 12x128 heads, FFN 8960, text cross-attention
+    over 512 context tokens) whose per-(step, layer) masks follow POLICY_PROFILE."""
+    hk, ck = policy_counts(12, 8960 // 8, n_layers)
+    return Config(name="wan13b_policy", dim=1536, n_heads=12, head_dim=128, ffn_dim=8960, grid=tuple(grid),
+                  heads_kept=hk, chunks_kept=ck, n_layers=n_layers, has_cross=1, ctx_len=512,
+                  xheads_kept=[list(h) for h in hk])
+
+
+def policy_small(n_layers: int = 12) -> Config:
+    """Tiny-shaped stack (d=256, 4x64 heads, FFN 1024, 2x8x8 tokens, cross-attention over 64
+    context tokens) with policy-shaped masks, small enough for the oracle's full denoise."""
+    hk, ck = policy_counts(4, 1024 // 8, n_layers)
+    return Config(name="policy_small", dim=256, n_heads=4, head_dim=64, ffn_dim=1024, grid=(2, 8, 8),
+                  heads_kept=hk, chunks_kept=ck, n_layers=n_layers, has_cross=1, ctx_len=64,
+                  xheads_kept=[list(h) for h in hk])
+
+
 def small_stack(n_layers: int = 4) -> Config:
     """Shrunken stack (d=256, 2x8x8 tokens, cross-attention) for end-to-end denoise checks."""
     cfg = tiny(n_layers=n_layers, has_cross=1, grid=(2, 8, 8))

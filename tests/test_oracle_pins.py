@@ -414,6 +414,30 @@ def test_flop_keep_reproduces_paper_cut():
     assert abs(f[0] - 3.8125e13) / 3.8125e13 < 1e-3
 
 
+def test_policy_shaped_masks_reproduce_the_paper_retention():
+    """The policy-shaped workload keeps the per-step FLOP fractions the paper reports for its
+    learned Wan-1.3B policy (Sec. 6) and has its described shape."""
+    cfg = synth.wan13b_policy()
+    N, d, dh = cfg.n_tokens, cfg.dim, cfg.head_dim
+    dense = O.block_flops(N, d, dh, cfg.n_heads, cfg.ffn_dim, cfg.n_heads, cfg.ctx_len)
+    ret = []
+    for s in range(4):
+        f = [O.block_flops(N, d, dh, cfg.heads_kept[s][l], 8 * cfg.chunks_kept[s][l], cfg.xheads_kept[s][l],
+                           cfg.ctx_len) for l in range(cfg.n_layers)]
+        ret.append(sum(f) / (cfg.n_layers * dense))
+    paper = GOLD["wan13b_step_retention"]["value"]
+    assert max(abs(a - b) for a, b in zip(ret, paper)) < 0.005, ret
+    assert abs(np.mean(ret) - GOLD["wan13b_final_flop_ratio"]["value"]) < 0.01
+    assert ret[0] > ret[1] and ret[3] > ret[2] and min(ret[0], ret[3]) > max(ret[1], ret[2])  # U shape
+    for s in range(4):
+        h, c = cfg.heads_kept[s], cfg.chunks_kept[s]
+        assert all(a >= b for a, b in zip(h, h[1:])) and all(a >= b for a, b in zip(c, c[1:]))  # depth
+        # attention keeps a smaller fraction than the FFN in the deepest layer
+        assert h[-1] / cfg.n_heads < c[-1] / cfg.n_chunks
+    assert cfg.heads_kept[1][-1] == 0 and cfg.heads_kept[2][-1] == 0       # deepest layer shut down
+    assert cfg.heads_kept[0][-1] > 0 and cfg.heads_kept[3][-1] > 0
+
+
 def test_denoise_with_all_blocks_off_is_geometric():
     cfg, W, LW, M, X = _problem()
     Mb = dict(M)
