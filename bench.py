@@ -35,7 +35,7 @@ import synth  # noqa: E402
 
 METRIC = "pruned-block TFLOP/s and % bf16 tensor peak; pruned/dense speedup vs ideal"
 KINDS = ("modulation", "adaln", "gemm_qkv", "qk_norm_rope", "attention", "gemm_o", "gemm_up", "gemm_down",
-         "cross", "other", "gather")
+         "cross", "other", "gather", "model")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -70,9 +70,15 @@ def _named_config(name: str):
         return synth.tiny()
     if name == "wan13b_policy":
         return synth.wan13b_policy()
+    if name == "wan13b_model":
+        return synth.wan13b_model()
     if name.startswith("sweep720:"):
         return synth.sweep720(float(name.split(":")[1]))
     raise SystemExit("unknown config " + name)
+
+
+def _is_model(cfg) -> bool:
+    return cfg.name.endswith("_model")
 
 
 def _policy_shaped(cfg) -> bool:
@@ -90,6 +96,11 @@ def workload_desc(cfg) -> str:
         fk = "/".join(str(8 * cfg.chunks_kept[s][0]) for s in range(cfg.n_steps))
     what = ("%d-layer %d-step denoise (dfs_denoise)" % (cfg.n_layers, cfg.n_steps) if cfg.n_layers > 1
             else "%d MoM steps per bench step" % cfg.n_steps)
+    if _is_model(cfg):
+        what = ("Wan-shaped model (patch embedding of a %dx%dx%dx%d latent, timestep MLP, head) around %d layers, "
+                "%d-step latent denoise (dfs_model_denoise, timesteps %s)"
+                % (cfg.latent_channels, cfg.grid[0], 2 * cfg.grid[1], 2 * cfg.grid[2], cfg.n_layers, cfg.n_steps,
+                   "/".join("%g" % t for t in synth.model_timesteps(cfg.n_steps))))
     cross = (", text cross-attention over %d context tokens (cross heads kept as self heads)" % cfg.ctx_len
              if cfg.has_cross else "")
     return ("%s-shaped pruned DiT block, %s: d=%d, %dx%d heads, FFN %d, %s=%d tokens, kept heads %s, "
@@ -130,6 +141,11 @@ def kernel_units(cfg):
                 u["cross"] += 4.0 * N * d * hc + 4.0 * N * cfg.ctx_len * hc
     if cfg.n_layers > 1:  # the stack's modulation GEMV runs once per step, not per layer
         u["modulation"] = cfg.n_steps * 6.0 * d * d * 2
+    if _is_model(cfg):    # model around the blocks, per step: token rows (4C wide) written by patchify and
+        # read by the embedding, the embedding's output, the head's LayerNorm in / out and GEMM input, the
+        # head's token rows and the latent read + written by the update (bf16)
+        C4 = 4 * cfg.latent_channels
+        u["model"] = cfg.n_steps * 2.0 * N * (2 * C4 + 4 * d + C4 + 2 * C4)
     bound = {k: ("tensor" if k.startswith("gemm") or k in ("attention", "cross") else "hbm") for k in KINDS}
     return u, bound
 
@@ -363,12 +379,33 @@ def run_ours(args):
         prob = None
     out = torch.empty_like(x)
     lat = x.clone()
+    model = _is_model(cfg)
+    if model:  # the model around the blocks: weights drawn on the device, latent from synth
+        g = torch.Generator(device="cuda")
+        g.manual_seed(7)
+        mw = {}
+        for k, shp in synth.model_shapes(cfg).items():
+            mw[k] = torch.empty(shp, device="cuda", dtype=torch.bfloat16)
+            mw[k].normal_(0.0, 0.02, generator=g)
+        for pl in (plan, dense_plan):
+            if pl is not None:
+                dfs.dfs_model_attach(pl, mw, cfg.latent_channels, cfg.freq_dim, stream)
+        del mw
+        latent0 = host.to_device(synth.make_latent(cfg))
+        lat = latent0.clone()
+        vbuf = torch.empty_like(latent0)
+        tsteps = synth.model_timesteps(T)
     weight_bytes, device_bytes = dfs.dfs_plan_memory(plan)
-    flops = [sum(dfs.dfs_plan_flops(plan, s, l) for l in range(L)) for s in range(T)]
+    # model: patch embedding and head GEMMs of every step count too (2 N (4C) d FLOPs each)
+    extra = 4.0 * cfg.n_tokens * 4 * cfg.latent_channels * cfg.dim if model else 0.0
+    flops = [sum(dfs.dfs_plan_flops(plan, s, l) for l in range(L)) + extra for s in range(T)]
     flops_step = sum(flops)
 
     def one_step():
-        if L == 1:
+        if model:
+            lat.copy_(latent0)
+            dfs.dfs_model_denoise(plan, lat, T, tsteps, stream)
+        elif L == 1:
             for s in range(T):
                 dfs.dfs_block_forward(plan, s, x, temb[s], out, stream)
         else:
@@ -442,6 +479,9 @@ def run_ours(args):
     bufs = (out, torch.empty_like(x)) if L > 1 else (out,)
 
     def run_step(pl, s):
+        if model:
+            dfs.dfs_model_forward(pl, s, latent0, tsteps[s], vbuf, stream)
+            return
         cur = x
         for l in range(L):
             dst = bufs[l % len(bufs)]
@@ -465,7 +505,7 @@ def run_ours(args):
         ref_ms, ref_flops, ref_desc = step_ms[0], flops[0], "step 0 (keeps every unit)"
     else:
         ref_ms = time_step(dense_plan, 0)
-        ref_flops = sum(dfs.dfs_plan_flops(dense_plan, 0, l) for l in range(L))
+        ref_flops = sum(dfs.dfs_plan_flops(dense_plan, 0, l) for l in range(L)) + extra
         ref_desc = "separate plan keeping every unit (%.2f ms)" % ref_ms
         dense_plan.close()
     ideal = [ref_flops / f for f in flops]
@@ -542,7 +582,8 @@ def main():
     ap.add_argument("--config", default="wan14b",
                     help="wan14b (default), wan13b, wan14b_cross, sweep720 (keep 1.0..0.5 as six steps), "
                          "sweep720:<ratio>, wan14b_x<L> (L-layer 4-step denoise with cross-attention), "
-                         "wan13b_policy (30-layer 4-step denoise, policy-shaped masks), tiny")
+                         "wan13b_policy (30-layer 4-step denoise, policy-shaped masks), wan13b_model (the same "
+                         "layers inside the Wan-shaped model on a latent video), tiny")
     ap.add_argument("--grid", default=None, help="override the latent grid T,H,W (smaller profiling cases)")
     ap.add_argument("--engine", choices=("compacted", "union"), default="compacted",
                     help="weights per (step, layer) compacted once (default), or one union super-model per "

@@ -151,6 +151,42 @@ dfs_status dfs_block_forward_noalloc(dfs_plan* plan, int step, int layer, const 
 dfs_status dfs_denoise(dfs_plan* plan, void* latents, int n_steps, const void* t_embs,
                        void* stream);
 
+/* The Wan-shaped model around the blocks -------------------------------------------
+ * (not specified by the paper, which prunes inside the blocks only; the wrapper lets the
+ * plan run complete denoising passes on a latent video.)  Readings: patch embedding of a
+ * latent video [C, F, H, W] (H = 2 grid_h, W = 2 grid_w, F = grid_t) in patches of
+ * 1 x 2 x 2, token n = (f grid_h + y) grid_w + x, feature c*4 + dy*2 + dx; x = patches
+ * patch_w^T + patch_b.  Timestep t -> e = [cos(t w_i), sin(t w_i)], w_i = 10000^(-i/(D/2));
+ * t_emb = t_w2 SiLU(t_w1 e + t_b1) + t_b2, which feeds every block's modulation (rounded to
+ * bf16) and the head.  Head: LN(x) (1 + head_mod[1] + t_emb) + head_mod[0] + t_emb, then
+ * v = . head_w^T + head_b, unpatched to [C, F, H, W].  bf16 DEVICE pointers, borrowed
+ * during dfs_model_attach only. */
+typedef struct {
+  int in_channels;                 /* latent channels C (16), even                    */
+  int freq_dim;                    /* sinusoid width D (256), multiple of 8, <= 8192   */
+  const void *patch_w, *patch_b;   /* [dim, 4 C], [dim]                                */
+  const void *t_w1, *t_b1;         /* [dim, D], [dim]                                  */
+  const void *t_w2, *t_b2;         /* [dim, dim], [dim]                                */
+  const void *head_mod;            /* [2, dim]: shift row, scale row                   */
+  const void *head_w, *head_b;     /* [4 C, dim], [4 C]                                */
+} dfs_model_weights;
+
+/* Copies the model weights into the plan and allocates the model's buffers (token rows
+ * [N, 4 C], the block input [N, dim], the timestep vectors).  May be called again to
+ * replace them.  Synchronises `stream`.  Errors: DFS_EINVAL, DFS_ENOMEM, DFS_ECUDA. */
+dfs_status dfs_model_attach(dfs_plan* plan, const dfs_model_weights* w, void* stream);
+
+/* One pass of the model at denoising step `step` (its structure) and timestep t (host):
+ * latent [C, F, H, W] bf16 device (read), v_out [C, F, H, W] bf16 device (written; may not
+ * alias latent).  Errors: DFS_EINVAL (no model attached, bad step, NULL, aliasing),
+ * DFS_ECUDA. */
+dfs_status dfs_model_forward(dfs_plan* plan, int step, const void* latent, float t, void* v_out, void* stream);
+
+/* Few-step sampling in latent space: for s in 0..n_steps-1, v = model(latent, step s,
+ * timesteps[s]) and latent <- latent + (1 / cfg.n_steps) v (block-gated layers skipped).
+ * latent [C, F, H, W] bf16 device, in/out; timesteps [n_steps] host floats. */
+dfs_status dfs_model_denoise(dfs_plan* plan, void* latent, int n_steps, const float* timesteps, void* stream);
+
 /* Test hooks ---------------------------------------------------------------------- */
 
 /* Index lists of I_t for (step, layer).  kind: 0 = retained head ids, 1 = retained FFN
@@ -223,7 +259,8 @@ typedef enum {
   DFS_K_CROSS = 8,        /* every kernel of the cross-attention branch                */
   DFS_K_OTHER = 9,        /* bias-only branches, Euler update, block-gate copies       */
   DFS_K_GATHER = 10,      /* union engine: per-forward FFN panel gathers from the union */
-  DFS_K_COUNT = 11
+  DFS_K_MODEL = 11,       /* model around the blocks: timestep MLP, patch embed, head   */
+  DFS_K_COUNT = 12
 } dfs_kernel_kind;
 
 /* Per-kernel timing of the forwards enqueued on this plan.  enable = 1 resets the

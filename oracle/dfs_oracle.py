@@ -32,6 +32,17 @@ authors' own engine for all of them):
   R7  FFN activation: GELU, tanh approximation.
   R8  a block whose block gate is 0 is the identity.
   R9  4-step sampler: x <- x + (1/T) * v with v the output of the last block.
+  R16 patch embedding of the Wan-shaped model around the blocks: latent video
+      [C, F, H, W], patches of 1 x 2 x 2; token n = (f*G_h + y)*G_w + x (the RoPE order),
+      feature k = c*4 + dy*2 + dx; x = patches W_p^T + b_p.
+  R17 timestep embedding: e = [cos(t w_i), sin(t w_i)], w_i = 10000^(-i/(D/2)),
+      i < D/2 (D = 256); t_emb = W_2 SiLU(W_1 e + b_1) + b_2.
+  R18 output head: LN(x) (no affine) * (1 + scale_h) + shift_h with
+      (shift_h, scale_h) = E_h + t_emb (a learned [2, d] table plus t_emb itself), then
+      v = y W_h^T + b_h, unpatched back to [C, F, H, W].
+  R19 latent sampler: the model predicts a velocity; z <- z + (1/T) v at each of the T
+      steps, step s fed with the host timestep t_s (1000 (1 - s/T): noise at s = 0, since
+      Sec. 3.1 puts tau = 0 at pure noise and tau = 1 at clean data).
 """
 from __future__ import annotations
 
@@ -46,6 +57,7 @@ __all__ = [
     "linear", "modulation", "layer_norm", "adaln", "rms_norm", "rope_pairs", "rope_angles",
     "apply_rope", "attention", "gelu_tanh", "block_forward_masked",
     "block_forward_compacted", "block_flops", "denoise", "MacCounter",
+    "patchify", "unpatchify", "timestep_embedding", "time_mlp", "model_forward", "model_denoise",
 ]
 
 
@@ -498,3 +510,72 @@ def denoise(cfg, shared, layers: List[Dict[str, np.ndarray]], masks, latents, t_
             h = block_forward_masked(cfg, shared, layers[l], masks, s, l, h, t_embs[s], ctx)
         x = x + (1.0 / cfg.n_steps) * h
     return x
+
+
+# ---------------------------------------------------------------------------------------
+# the Wan-shaped model around the blocks (R16-R19)
+# ---------------------------------------------------------------------------------------
+
+PATCH = (1, 2, 2)
+
+
+def patchify(latent) -> np.ndarray:
+    """[C, F, H, W] -> [F * H/2 * W/2, 4 C] (R16): the 2 x 2 patch at (f, y, x) becomes token
+    (f * H/2 + y) * W/2 + x with feature c*4 + dy*2 + dx = latent[c, f, 2y + dy, 2x + dx]."""
+    C, F, H, W = latent.shape
+    gh, gw = H // 2, W // 2
+    out = np.empty((F * gh * gw, 4 * C), dtype=latent.dtype)
+    for c in range(C):
+        for dy in range(2):
+            for dx in range(2):
+                out[:, c * 4 + dy * 2 + dx] = latent[c, :, dy::2, dx::2].reshape(-1)
+    return out
+
+
+def unpatchify(tokens, shape) -> np.ndarray:
+    """Inverse of ``patchify`` for a latent of the given [C, F, H, W] shape."""
+    C, F, H, W = shape
+    out = np.empty(shape, dtype=tokens.dtype)
+    for c in range(C):
+        for dy in range(2):
+            for dx in range(2):
+                out[c, :, dy::2, dx::2] = tokens[:, c * 4 + dy * 2 + dx].reshape(F, H // 2, W // 2)
+    return out
+
+
+def timestep_embedding(t: float, dim: int) -> np.ndarray:
+    """[cos(t w), sin(t w)] with w_i = 10000^(-i / (dim/2)) (R17)."""
+    half = dim // 2
+    w = 10000.0 ** (-np.arange(half, dtype=np.float64) / half)
+    return np.concatenate([np.cos(t * w), np.sin(t * w)])
+
+
+def time_mlp(mw, t: float) -> np.ndarray:
+    """t_emb = W_2 SiLU(W_1 e + b_1) + b_2 (R17)."""
+    e = timestep_embedding(t, mw["t_w1"].shape[1])
+    h = mw["t_w1"] @ e + mw["t_b1"]
+    h = h / (1.0 + np.exp(-h))
+    return mw["t_w2"] @ h + mw["t_b2"]
+
+
+def model_forward(cfg, shared, layers, mw, masks, step: int, latent, t: float, ctx=None, want: bool = False):
+    """One pass of the Wan-shaped model at denoising step `step` (R16-R18): patch embedding,
+    every block with its step-`step` structure (masked-dense form), output head; returns the
+    velocity in latent layout [C, F, H, W]."""
+    t_emb = time_mlp(mw, t)
+    x = linear(patchify(latent), mw["patch_w"], mw["patch_b"])
+    for l in range(cfg.n_layers):
+        x = block_forward_masked(cfg, shared, layers[l], masks, step, l, x, t_emb, ctx)
+    shift = mw["head_mod"][0] + t_emb
+    scale = mw["head_mod"][1] + t_emb
+    y = adaln(x, shift, scale, cfg.ln_eps)
+    v = unpatchify(linear(y, mw["head_w"], mw["head_b"]), latent.shape)
+    return (v, {"t_emb": t_emb, "x_last": x}) if want else v
+
+
+def model_denoise(cfg, shared, layers, mw, masks, latent, timesteps, ctx=None):
+    """T steps of z <- z + (1/T) v(z, t_s) with step s's structure (R19)."""
+    z = latent.copy()
+    for s, t in enumerate(timesteps):
+        z = z + (1.0 / cfg.n_steps) * model_forward(cfg, shared, layers, mw, masks, s, z, t, ctx)
+    return z

@@ -125,6 +125,14 @@ struct dfs_plan {
   bf16* ffn_down_s = nullptr;  //   union at every forward ([f_s, d] and [d, f_s], largest step)
   long long bytes_total = 0, bytes_weights = 0;
   std::vector<void*> temps;    // device buffers needed only during plan creation
+  // model around the blocks (dfs_model_attach)
+  bool has_model = false;
+  int mC = 0, mD = 0;
+  bf16 *m_patch_w = nullptr, *m_patch_b = nullptr, *m_t_w1 = nullptr, *m_t_b1 = nullptr, *m_t_w2 = nullptr,
+       *m_t_b2 = nullptr, *m_head_mod = nullptr, *m_head_w = nullptr, *m_head_b = nullptr;
+  bf16 *m_tok = nullptr, *m_x0 = nullptr, *m_vtok = nullptr, *m_temb = nullptr;
+  float *m_freq = nullptr, *m_h1 = nullptr, *m_temb_f = nullptr, *m_hm = nullptr;
+  dfs::GemmArgs g_embed, g_head;
   bf16* w_t = nullptr;
   bf16* b_t = nullptr;
   dfs::RopeTables rope{};
@@ -940,6 +948,121 @@ dfs_status dfs_denoise(dfs_plan* P, void* latents, int n_steps, const void* t_em
       ping ^= 1;
     }
     DFS_LAUNCH(DFS_K_OTHER, dfs::launch_euler(lat, cur, 1.f / P->cfg.n_steps, static_cast<long long>(P->N) * d, st));
+  }
+  return DFS_OK;
+}
+
+// ------------------------------------------------------------------ model around the blocks
+
+}  // extern "C"
+
+namespace {
+
+// One pass of the model on `lat` at step s with host timestep t: the timestep MLP, patch
+// embedding, every layer of step s, the head; leaves the velocity token rows in m_vtok.
+dfs_status model_pass(dfs_plan* P, int s, const bf16* lat, float t, cudaStream_t st) {
+  const dfs_config& c = P->cfg;
+  const int d = c.dim, C = P->mC;
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_timestep_freq(P->m_freq, static_cast<double>(t), P->mD, st));
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_gemv(P->m_h1, nullptr, P->m_t_w1, P->m_t_b1, P->m_freq, d, P->mD, 0, st));
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_gemv(P->m_temb_f, P->m_temb, P->m_t_w2, P->m_t_b2, P->m_h1, d, d, 1, st));
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_patchify(P->m_tok, lat, C, c.grid_t, c.grid_h, c.grid_w, st));
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_gemm(P->g_embed, P->num_sms, st));
+  float* base = P->mod_base + 6LL * d * s;
+  DFS_LAUNCH(DFS_K_MODULATION, dfs::launch_modulation(base, P->w_t, P->b_t, nullptr, P->m_temb, 6 * d, d, st));
+  const bf16* cur = P->m_x0;
+  int ping = 0;
+  for (int l = 0; l < P->L; ++l) {
+    if (!P->block_gate[static_cast<size_t>(s) * P->L + l]) continue;
+    DFS_LAUNCH(DFS_K_MODULATION, dfs::launch_add_table(P->mod, base, P->lc[l].emod, 6 * d, st));
+    bf16* dst = P->act[ping];
+    dfs_status e = forward_impl(P, s, l, cur, dst, st);
+    if (e) return e;
+    cur = dst;
+    ping ^= 1;
+  }
+  // head: (shift, scale) = head_mod + t_emb; LN + modulate into xm; v tokens = xm head_w^T + b
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_add_table(P->m_hm, P->m_temb_f, P->m_head_mod, d, st));
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_add_table(P->m_hm + d, P->m_temb_f, P->m_head_mod + d, d, st));
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_row_norm(P->xm, cur, 0, P->N, d, P->m_hm + d, 1.f, P->m_hm, c.ln_eps, st));
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_gemm(P->g_head, P->num_sms, st));
+  return DFS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+dfs_status dfs_model_attach(dfs_plan* P, const dfs_model_weights* w, void* stream) {
+  if (!P || !w) return fail(DFS_EINVAL, "NULL plan or weights");
+  const void* req[] = {w->patch_w, w->patch_b, w->t_w1, w->t_b1, w->t_w2, w->t_b2, w->head_mod, w->head_w, w->head_b};
+  for (const void* q : req)
+    if (!q) return fail(DFS_EINVAL, "NULL model weight pointer");
+  if (w->in_channels < 2 || w->in_channels % 2 != 0 || w->in_channels > 1024)
+    return fail(DFS_EINVAL, "in_channels must be even, 2..1024");
+  if (w->freq_dim < 8 || w->freq_dim % 8 != 0 || w->freq_dim > 8192)
+    return fail(DFS_EINVAL, "freq_dim must be a multiple of 8 in 8..8192");
+  if (P->has_model) return fail(DFS_EUNSUPPORTED, "a model is already attached to this plan");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const long long d = P->cfg.dim, C = w->in_channels, D = w->freq_dim, N = P->N, p4 = 4 * C;
+  P->mC = static_cast<int>(C);
+  P->mD = static_cast<int>(D);
+  dfs_status e;
+  struct Cp { bf16** dst; const void* src; long long n; };
+  const Cp cps[] = {{&P->m_patch_w, w->patch_w, d * p4}, {&P->m_patch_b, w->patch_b, d}, {&P->m_t_w1, w->t_w1, d * D},
+                    {&P->m_t_b1, w->t_b1, d}, {&P->m_t_w2, w->t_w2, d * d}, {&P->m_t_b2, w->t_b2, d},
+                    {&P->m_head_mod, w->head_mod, 2 * d}, {&P->m_head_w, w->head_w, p4 * d},
+                    {&P->m_head_b, w->head_b, p4}};
+  for (const Cp& q : cps) {
+    if ((e = alloc_weights(P, q.dst, q.n))) return e;
+    DFS_CK(cudaMemcpyAsync(*q.dst, q.src, 2 * q.n, cudaMemcpyDeviceToDevice, st));
+  }
+  if ((e = alloc_n(P, &P->m_tok, N * p4)) || (e = alloc_n(P, &P->m_x0, N * d)) || (e = alloc_n(P, &P->m_vtok, N * p4)) ||
+      (e = alloc_n(P, &P->m_temb, d)) || (e = alloc_n(P, &P->m_freq, D)) || (e = alloc_n(P, &P->m_h1, d)) ||
+      (e = alloc_n(P, &P->m_temb_f, d)) || (e = alloc_n(P, &P->m_hm, 2 * d)))
+    return e;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, P->m_tok, p4, N, p4, 64, 128) || !make_map(&mb, P->m_patch_w, p4, d, p4, 64, dfs::kGemmBRows))
+    return fail(DFS_ECUDA, "tensor map (patch embedding) failed");
+  P->g_embed = gemm_args(P, ma, mb, static_cast<int>(N), static_cast<int>(d), static_cast<int>(p4), dfs::kEpiBias,
+                         P->m_patch_b);
+  P->g_embed.out = P->m_x0; P->g_embed.ldo = d;
+  if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, P->m_head_w, d, p4, d, 64, dfs::kGemmBRows))
+    return fail(DFS_ECUDA, "tensor map (head) failed");
+  P->g_head = gemm_args(P, ma, mb, static_cast<int>(N), static_cast<int>(p4), static_cast<int>(d), dfs::kEpiBias,
+                        P->m_head_b);
+  P->g_head.out = P->m_vtok; P->g_head.ldo = p4;
+  DFS_CK(cudaStreamSynchronize(st));
+  P->has_model = true;
+  return DFS_OK;
+}
+
+dfs_status dfs_model_forward(dfs_plan* P, int step, const void* latent, float t, void* v_out, void* stream) {
+  if (!P || !latent || !v_out) return fail(DFS_EINVAL, "NULL plan, latent or v_out");
+  if (!P->has_model) return fail(DFS_EINVAL, "no model attached (dfs_model_attach)");
+  if (latent == v_out) return fail(DFS_EINVAL, "latent and v_out must not alias");
+  if (step < 0 || step >= P->T) return fail(DFS_EINVAL, "step %d out of range [0, %d)", step, P->T);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  dfs_status e = model_pass(P, step, static_cast<const bf16*>(latent), t, st);
+  if (e) return e;
+  const dfs_config& c = P->cfg;
+  DFS_LAUNCH(DFS_K_MODEL, dfs::launch_unpatchify(static_cast<bf16*>(v_out), nullptr, P->m_vtok, 1.f, P->mC, c.grid_t,
+                                                 c.grid_h, c.grid_w, st));
+  return DFS_OK;
+}
+
+dfs_status dfs_model_denoise(dfs_plan* P, void* latent, int n_steps, const float* timesteps, void* stream) {
+  if (!P || !latent || !timesteps) return fail(DFS_EINVAL, "NULL plan, latent or timesteps");
+  if (!P->has_model) return fail(DFS_EINVAL, "no model attached (dfs_model_attach)");
+  if (n_steps < 1 || n_steps > P->T) return fail(DFS_EINVAL, "n_steps must be in 1..%d", P->T);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const dfs_config& c = P->cfg;
+  bf16* lat = static_cast<bf16*>(latent);
+  for (int s = 0; s < n_steps; ++s) {
+    dfs_status e = model_pass(P, s, lat, timesteps[s], st);
+    if (e) return e;
+    DFS_LAUNCH(DFS_K_MODEL, dfs::launch_unpatchify(lat, lat, P->m_vtok, 1.f / c.n_steps, P->mC, c.grid_t, c.grid_h,
+                                                   c.grid_w, st));
   }
   return DFS_OK;
 }

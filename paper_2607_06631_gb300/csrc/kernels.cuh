@@ -133,6 +133,19 @@ cudaError_t launch_to_f32(float* out, const bf16* in, int n, cudaStream_t s);
 // Waits (bounded) on an mbarrier that nothing completes; sets *err to kErrTimeout.
 cudaError_t launch_wait_selftest(int* err, cudaStream_t s);
 
+// Model around the blocks (model.cu).
+// e[i] = cos(t w_i), e[dim/2 + i] = sin(t w_i), w_i = 10000^(-i / (dim/2)); e fp32 [dim].
+cudaError_t launch_timestep_freq(float* e, double t, int dim, cudaStream_t s);
+// out[r] = sum_c W[r, c] f(in[c]) + b[r] for r < rows, f = SiLU when silu_in, else identity;
+// W bf16 [rows, cols] (cols % 8 == 0), in fp32 [cols]; out_f32 / out_bf16 may be null.
+cudaError_t launch_gemv(float* out_f32, bf16* out_bf16, const bf16* W, const bf16* b, const float* in, int rows,
+                        int cols, int silu_in, cudaStream_t s);
+// tok[n, 4c + 2dy + dx] = lat[c, f, 2y + dy, 2x + dx], n = (f gh + y) gw + x; lat [C, F, 2gh, 2gw].
+cudaError_t launch_patchify(bf16* tok, const bf16* lat, int C, int F, int gh, int gw, cudaStream_t s);
+// out[c, f, 2y + dy, 2x + dx] = (base ? base[same] : 0) + dt * tok[n, 4c + 2dy + dx] (out may alias base).
+cudaError_t launch_unpatchify(bf16* out, const bf16* base, const bf16* tok, float dt, int C, int F, int gh, int gw,
+                              cudaStream_t s);
+
 // K8: x = x + dt * v (bf16, n elements, n % 8 == 0).
 cudaError_t launch_euler(bf16* x, const bf16* v, float dt, long long n, cudaStream_t s);
 

@@ -25,10 +25,11 @@ EXPORTED = ("dfs_plan_create", "dfs_block_forward", "dfs_block_forward_layer", "
             "dfs_denoise", "dfs_plan_indices", "dfs_plan_panel", "dfs_plan_union_panel", "dfs_plan_memory",
             "dfs_plan_flops", "dfs_plan_workspace",
             "dfs_plan_sync", "dfs_selftest_wait_timeout", "dfs_plan_profile", "dfs_plan_profile_read", "dfs_gates_from_soft_masks",
+            "dfs_model_attach", "dfs_model_forward", "dfs_model_denoise",
             "dfs_plan_destroy", "dfs_last_error")
 
 KERNEL_KINDS = ("modulation", "adaln", "gemm_qkv", "qk_norm_rope", "attention", "gemm_o", "gemm_up",
-                "gemm_down", "cross", "other", "gather")
+                "gemm_down", "cross", "other", "gather", "model")
 
 PANELS = {"wqkv": 0, "bqkv": 1, "gq": 2, "gk": 3, "wo": 4, "w_up": 5, "b_up": 6, "w_down": 7,
           "cwq": 8, "cbq": 9, "cwkv": 10, "cbkv": 11, "cgq": 12, "cgk": 13, "cwo": 14}
@@ -66,6 +67,14 @@ class dfs_masks(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in ("block_gate", "head_gate", "xhead_gate", "ffn_gate")]
 
 
+MODEL_FIELDS = ("patch_w", "patch_b", "t_w1", "t_b1", "t_w2", "t_b2", "head_mod", "head_w", "head_b")
+
+
+class dfs_model_weights(ctypes.Structure):
+    _fields_ = [("in_channels", ctypes.c_int), ("freq_dim", ctypes.c_int)] + \
+               [(n, ctypes.c_void_p) for n in MODEL_FIELDS]
+
+
 _lib = None
 
 
@@ -96,6 +105,9 @@ def lib() -> ctypes.CDLL:
         L.dfs_plan_profile.argtypes = [vp, i32]
         L.dfs_plan_profile_read.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_double), i64p]
         L.dfs_gates_from_soft_masks.argtypes = [i32, i32, i32, i32, vp, vp]
+        L.dfs_model_attach.argtypes = [vp, ctypes.POINTER(dfs_model_weights), vp]
+        L.dfs_model_forward.argtypes = [vp, i32, vp, ctypes.c_float, vp, vp]
+        L.dfs_model_denoise.argtypes = [vp, vp, i32, vp, vp]
         L.dfs_plan_destroy.argtypes = [vp]
         L.dfs_plan_destroy.restype = None
         L.dfs_last_error.restype = ctypes.c_char_p
@@ -233,6 +245,24 @@ def dfs_block_forward_noalloc(plan, step: int, layer: int, x, t_emb, out, stream
 
 def dfs_denoise(plan, latents, n_steps: int, t_embs, stream=None):
     _check(lib().dfs_denoise(_h(plan), _ptr(latents), n_steps, _ptr(t_embs), _stream(stream)))
+
+
+def dfs_model_attach(plan, weights: Dict[str, Any], in_channels: int = 16, freq_dim: int = 256, stream=None):
+    """weights: device buffers keyed like dfs_model_weights (bf16)."""
+    w = dfs_model_weights()
+    w.in_channels, w.freq_dim = in_channels, freq_dim
+    for f in MODEL_FIELDS:
+        setattr(w, f, _ptr(weights.get(f)))
+    _check(lib().dfs_model_attach(_h(plan), ctypes.byref(w), _stream(stream)))
+
+
+def dfs_model_forward(plan, step: int, latent, t: float, v_out, stream=None):
+    _check(lib().dfs_model_forward(_h(plan), step, _ptr(latent), float(t), _ptr(v_out), _stream(stream)))
+
+
+def dfs_model_denoise(plan, latent, n_steps: int, timesteps: Sequence[float], stream=None):
+    ts = np.ascontiguousarray(timesteps, dtype=np.float32)
+    _check(lib().dfs_model_denoise(_h(plan), _ptr(latent), n_steps, ts.ctypes.data, _stream(stream)))
 
 
 def dfs_plan_indices(plan, step: int, layer: int, kind) -> np.ndarray:

@@ -75,6 +75,8 @@ class Config:
     qk_norm_mode: int = 0
     block_gate: Optional[List[List[int]]] = None  # [n_steps][n_layers]; None -> all ones
     engine: int = 0        # how the library holds the weights: 0 per-step copies, 1 union
+    latent_channels: int = 16   # Wan-shaped model around the blocks: latent video channels
+    freq_dim: int = 256         # and timestep-sinusoid width
 
     @property
     def n_tokens(self) -> int:
@@ -212,6 +214,27 @@ def small_stack(n_layers: int = 4) -> Config:
     return cfg
 
 
+def tiny_model(n_layers: int = 4) -> Config:
+    """Tiny-shaped model (d=256, 4x64 heads, FFN 1024, cross-attention over 64 context
+    tokens) on a 16 x 2 x 16 x 16 latent video (2 x 8 x 8 = 128 tokens)."""
+    cfg = tiny(n_layers=n_layers, has_cross=1, grid=(2, 8, 8))
+    cfg.name = "tiny_model"
+    cfg.ctx_len = 64
+    return cfg
+
+
+def wan13b_model() -> Config:
+    """The 30-layer Wan-1.3B-shaped policy stack inside the model (latent 16 x 21 x 60 x 104)."""
+    cfg = wan13b_policy()
+    cfg.name = "wan13b_model"
+    return cfg
+
+
+def model_timesteps(n_steps: int = 4) -> List[float]:
+    """Host timesteps fed to the model's sinusoid at each step: 1000 (1 - s/T)."""
+    return [1000.0 * (1.0 - s / n_steps) for s in range(n_steps)]
+
+
 # ---------------------------------------------------------------------------------------
 # seeded draws
 # ---------------------------------------------------------------------------------------
@@ -325,6 +348,26 @@ def make_activations(cfg: Config, seed_tag: str = "") -> Dict[str, np.ndarray]:
     if cfg.has_cross:
         out["ctx"] = normal_bits((cfg.ctx_len, d), 1.0, 0.0, cfg.name + seed_tag, "ctx")
     return out
+
+
+MODEL_KEYS = ("patch_w", "patch_b", "t_w1", "t_b1", "t_w2", "t_b2", "head_mod", "head_w", "head_b")
+
+
+def model_shapes(cfg: Config) -> Dict[str, tuple]:
+    d, p = cfg.dim, 4 * cfg.latent_channels
+    return {"patch_w": (d, p), "patch_b": (d,), "t_w1": (d, cfg.freq_dim), "t_b1": (d,),
+            "t_w2": (d, d), "t_b2": (d,), "head_mod": (2, d), "head_w": (p, d), "head_b": (p,)}
+
+
+def make_model_weights(cfg: Config, seed_tag: str = "") -> Dict[str, np.ndarray]:
+    """Weights of the model around the blocks, all ~ N(0, 0.02) as bf16 bits."""
+    return {k: normal_bits(shp, 0.02, 0.0, cfg.name + seed_tag, "model", k) for k, shp in model_shapes(cfg).items()}
+
+
+def make_latent(cfg: Config, seed_tag: str = "") -> np.ndarray:
+    """Latent video [C, F, H, W] ~ N(0, 1) as bf16 bits (H, W = twice the token grid)."""
+    F, gh, gw = cfg.grid
+    return normal_bits((cfg.latent_channels, F, 2 * gh, 2 * gw), 1.0, 0.0, cfg.name + seed_tag, "latent")
 
 
 def make_problem(cfg: Config, seed_tag: str = ""):

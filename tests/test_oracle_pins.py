@@ -446,6 +446,84 @@ def test_denoise_with_all_blocks_off_is_geometric():
     np.testing.assert_allclose(out, X["x"] * (1 + 1 / GOLD["n_steps"]["value"]) ** 4, rtol=1e-14)
 
 
+# --------------------------------------------------------------------------- model around the blocks (R16-R19)
+
+def test_patchify_places_each_latent_element_by_hand():
+    C, F, H, W = 2, 2, 4, 6
+    lat = np.zeros((C, F, H, W))
+    for c in range(C):
+        for f in range(F):
+            for y in range(H):
+                for x in range(W):
+                    lat[c, f, y, x] = 1000 * c + 100 * f + 10 * y + x
+    tok = O.patchify(lat)
+    assert tok.shape == (F * 2 * 3, 4 * C)
+    # the patch at frame 1, patch row 1, patch column 1 (token grid 2 x 3): latent rows 2, 3 and
+    # columns 2, 3; token (1 * 2 + 1) * 3 + 1 = 10; features c*4 + dy*2 + dx
+    n = (1 * 2 + 1) * 3 + 1
+    assert tok[n].tolist() == [100 + 20 + 2, 100 + 20 + 3, 100 + 30 + 2, 100 + 30 + 3,
+                               1100 + 20 + 2, 1100 + 20 + 3, 1100 + 30 + 2, 1100 + 30 + 3]
+    np.testing.assert_array_equal(O.unpatchify(tok, lat.shape), lat)
+
+
+def test_timestep_embedding_textbook_values():
+    np.testing.assert_array_equal(O.timestep_embedding(0.0, 8), [1, 1, 1, 1, 0, 0, 0, 0])
+    e = O.timestep_embedding(1.0, 4)      # w = [1, 10000^-0.5]
+    np.testing.assert_allclose(e, [math.cos(1), math.cos(0.01), math.sin(1), math.sin(0.01)], rtol=1e-15)
+    e = O.timestep_embedding(750.0, 256)
+    np.testing.assert_allclose(e[:128] ** 2 + e[128:] ** 2, 1.0, rtol=1e-12)
+
+
+def test_time_mlp_silu():
+    d, D = 4, 8
+    mw = {"t_w1": np.zeros((d, D)), "t_b1": np.array([0.0, 1.0, -1.0, 3.0]), "t_w2": np.eye(d),
+          "t_b2": np.array([0.5, 0, 0, 0])}
+    sig = lambda v: 1 / (1 + math.exp(-v))
+    np.testing.assert_allclose(O.time_mlp(mw, 123.0), [0.5, sig(1.0), -sig(-1.0), 3 * sig(3.0)], rtol=1e-15)
+
+
+def _model_problem(seed_tag=""):
+    cfg = synth.tiny_model(n_layers=2)
+    cfg.grid = (2, 4, 4)
+    sh, L, M, A = synth.make_problem(cfg, seed_tag)
+    mw = synth.widen(synth.make_model_weights(cfg, seed_tag))
+    lat = synth.bits_to_f64(synth.make_latent(cfg, seed_tag))
+    return cfg, synth.widen(sh), synth.widen(L), M, synth.widen(A), mw, lat
+
+
+def test_model_head_reads_only_its_bias_when_its_weights_vanish():
+    cfg, W, LW, M, X, mw, lat = _model_problem()
+    mw = dict(mw)
+    mw["head_w"] = np.zeros_like(mw["head_w"])
+    v = O.model_forward(cfg, W, LW, mw, M, 1, lat, 750.0, X["ctx"])
+    want = O.unpatchify(np.tile(mw["head_b"], (cfg.n_tokens, 1)), lat.shape)
+    np.testing.assert_allclose(v, want, rtol=0, atol=0)
+
+
+def test_model_blocks_off_leave_the_embedded_patches():
+    """With every block gated off the head sees the patch embedding itself."""
+    cfg, W, LW, M, X, mw, lat = _model_problem()
+    Mb = dict(M)
+    Mb["block_gate"] = np.zeros_like(M["block_gate"])
+    v, it = O.model_forward(cfg, W, LW, mw, Mb, 0, lat, 1000.0, X["ctx"], want=True)
+    np.testing.assert_array_equal(it["x_last"], O.patchify(lat) @ mw["patch_w"].T + mw["patch_b"])
+    np.testing.assert_allclose(it["t_emb"], O.time_mlp(mw, 1000.0))
+
+
+def test_model_denoise_sums_the_step_velocities():
+    cfg, W, LW, M, X, mw, lat = _model_problem()
+    ts = synth.model_timesteps(4)
+    assert ts == [1000.0, 750.0, 500.0, 250.0]
+    z = lat.copy()
+    vs = []
+    for s in range(4):
+        v = O.model_forward(cfg, W, LW, mw, M, s, z, ts[s], X["ctx"])
+        vs.append(v)
+        z = z + v / 4
+    np.testing.assert_allclose(O.model_denoise(cfg, W, LW, mw, M, lat, ts, X["ctx"]), lat + sum(vs) / 4,
+                               rtol=1e-12, atol=1e-12)
+
+
 # --------------------------------------------------------------------------- input generator
 
 def test_bf16_rounding_matches_torch():
