@@ -302,27 +302,10 @@ def run_reference(args):
 # ------------------------------------------------------------------------------ our arm
 
 def device_stack(cfg, seed: int = 20260706):
-    """Random-init weights of a multi-layer stack drawn directly on the device (torch
-    generator; N(0, 0.02) weights, 1 + 0.1 N(0, 1) norm scales): tens of GB would take
-    minutes through the host generator.  Masks, inputs and text context come from synth."""
-    import torch
+    """Random-init stack weights drawn on the device (host.random_device_stack); masks,
+    inputs and text context come from synth."""
     from paper_2607_06631_gb300 import host
-    g = torch.Generator(device="cuda")
-    g.manual_seed(seed)
-
-    def draw(shape, std, mean=0.0):
-        t = torch.empty(shape, device="cuda", dtype=torch.bfloat16)
-        t.normal_(mean, std, generator=g)
-        return t
-    layers = []
-    for _ in range(cfg.n_layers):
-        lw = {}
-        for k, shp in synth.layer_shapes(cfg).items():
-            scale = k in ("gq", "gk", "cgq", "cgk", "cln_w")
-            lw[k] = draw(shp, 0.1 if scale else 0.02, 1.0 if scale else 0.0)
-        layers.append(lw)
-    d = cfg.dim
-    w_t, b_t = draw((6 * d, d), 0.02), draw((6 * d,), 0.02)
+    layers, w_t, b_t = host.random_device_stack(cfg, seed)
     acts = synth.make_activations(cfg)
     x = host.to_device(acts["x"])
     temb = host.to_device(acts["t_emb"])

@@ -98,7 +98,11 @@ typedef struct {
  *   w_t [6*dim, dim], b_t [6*dim]: shared adaLN linear (bf16 device, borrowed).
  *   ctx [ctx_len, dim] bf16 device or NULL when has_cross == 0 (borrowed).
  * Synchronises `stream` before returning.  On failure *out is NULL and everything
- * allocated so far is freed.  Errors: DFS_EINVAL, DFS_ENOMEM, DFS_ECUDA. */
+ * allocated so far is freed.  Errors: DFS_EINVAL, DFS_ENOMEM, DFS_ECUDA.
+ * Host-side fault injection for tests, read here from the environment: DFS_FAULT_ALLOC=n
+ * makes the plan's n-th device allocation fail (DFS_ENOMEM); DFS_FAULT_LAUNCH=n makes the
+ * plan's n-th kernel launch (counted over its forwards) be skipped and reported as
+ * DFS_ECUDA.  Every kernel launch is wrapped in an NVTX range named "dfs <kind>". */
 dfs_status dfs_plan_create(const dfs_config* cfg, const dfs_layer_weights* layers /*[n_layers]*/,
                            const void* w_t, const void* b_t, const dfs_masks* masks,
                            const void* ctx, void* stream, dfs_plan** out);

@@ -12,6 +12,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/dfs.h"
 #include "kernels.cuh"
 
@@ -154,6 +156,7 @@ struct dfs_plan {
   std::vector<void*> allocs;
   int last_step = -1, last_layer = -1;
   int fault_alloc = -1, n_alloc = 0;  // host-side fault injection (DFS_FAULT_ALLOC=n)
+  long long fault_launch = -1, n_launch = 0;  // (DFS_FAULT_LAUNCH=n: the n-th launch fails)
   // per-kernel profiling: event pairs recorded around launches while prof_on
   bool prof_on = false;
   std::vector<cudaEvent_t> ev;  // pool, pairs (2i, 2i+1)
@@ -220,16 +223,25 @@ void free_plan(dfs_plan* P) {
 
 // ------------------------------------------------------------------ per-kernel profiling
 
-// Brackets one kernel launch: records an event before and after it on `st` while
-// profiling is on, and counts the launch.
+const char* const kKindNames[DFS_K_COUNT] = {"dfs modulation", "dfs adaln", "dfs gemm_qkv", "dfs qk_norm_rope",
+                                             "dfs attention", "dfs gemm_o", "dfs gemm_up", "dfs gemm_down",
+                                             "dfs cross", "dfs other", "dfs gather", "dfs model"};
+
+// Brackets one kernel launch: an NVTX range named by its kind (seen by Nsight tools, free
+// without one), an event before and after it on `st` while profiling is on, and the launch
+// count.  `inject` is set for the launch DFS_FAULT_LAUNCH names, which is then skipped and
+// reported as a failed launch (host-side fault injection; nothing reaches the GPU).
 struct ProfScope {
   dfs_plan* P;
   int kind;
   cudaStream_t st;
   int pair = -1;
+  bool inject = false;
   ProfScope(dfs_plan* p, int k, cudaStream_t s) : P(p), kind(k), st(s) {
+    nvtxRangePushA(kKindNames[kind]);
     ++P->launches[kind];
-    if (!P->prof_on) return;
+    inject = ++P->n_launch == P->fault_launch;
+    if (!P->prof_on || inject) return;
     if (2 * P->ev_used + 2 > P->ev.size()) {
       cudaEvent_t a, b;
       if (cudaEventCreate(&a) != cudaSuccess) return;
@@ -244,13 +256,15 @@ struct ProfScope {
   }
   ~ProfScope() {
     if (pair >= 0) cudaEventRecord(P->ev[2 * pair + 1], st);
+    nvtxRangePop();
   }
 };
 
-#define DFS_LAUNCH(kind, expr)                \
-  do {                                        \
-    ProfScope prof_(P, (kind), st);           \
-    DFS_CK(expr);                             \
+#define DFS_LAUNCH(kind, expr)                                                                  \
+  do {                                                                                          \
+    ProfScope prof_(P, (kind), st);                                                             \
+    if (prof_.inject) return fail(DFS_ECUDA, "injected launch failure at launch %lld", P->n_launch); \
+    DFS_CK(expr);                                                                               \
   } while (0)
 
 // ------------------------------------------------------------------ validation (host only)
@@ -886,6 +900,7 @@ dfs_status dfs_plan_create(const dfs_config* cfg, const dfs_layer_weights* layer
   P->N = cfg->grid_t * cfg->grid_h * cfg->grid_w;
   P->block_gate.assign(masks->block_gate, masks->block_gate + static_cast<size_t>(P->T) * P->L);
   if (const char* f = getenv("DFS_FAULT_ALLOC")) P->fault_alloc = atoi(f);
+  if (const char* f = getenv("DFS_FAULT_LAUNCH")) P->fault_launch = atoll(f);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   e = create_impl(P, layers, w_t, b_t, masks, ctx, st);
   if (e) {

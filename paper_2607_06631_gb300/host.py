@@ -90,3 +90,27 @@ class DeviceProblem:
         """Drops the full weights once the plan holds its compacted copies."""
         self.layers = None
         self.w_t = self.b_t = None
+
+
+def random_device_stack(cfg, seed: int = 20260706):
+    """Random-init weights of a multi-layer stack drawn directly on the device (torch's
+    generator; N(0, 0.02) weights and biases, 1 + 0.1 N(0, 1) norm scales, the shapes of
+    synth.layer_shapes): tens of GB would take minutes through the host generator.
+    Returns (layers [per-layer dicts of bf16 tensors], w_t, b_t)."""
+    import synth
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+
+    def draw(shape, std, mean=0.0):
+        t = torch.empty(shape, device="cuda", dtype=torch.bfloat16)
+        t.normal_(mean, std, generator=g)
+        return t
+    layers = []
+    for _ in range(cfg.n_layers):
+        lw = {}
+        for k, shp in synth.layer_shapes(cfg).items():
+            scale = k in ("gq", "gk", "cgq", "cgk", "cln_w")
+            lw[k] = draw(shp, 0.1 if scale else 0.02, 1.0 if scale else 0.0)
+        layers.append(lw)
+    d = cfg.dim
+    return layers, draw((6 * d, d), 0.02), draw((6 * d,), 0.02)

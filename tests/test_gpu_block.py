@@ -158,6 +158,32 @@ def test_injected_allocation_failure(monkeypatch):
     prob.create_plan()
 
 
+def test_injected_launch_failure_is_reported_and_the_plan_recovers(monkeypatch):
+    """DFS_FAULT_LAUNCH=n skips the plan's n-th launch and reports it: the forward that hits
+    it returns DFS_ECUDA and leaves `out` untouched; the next forward is correct."""
+    import torch
+    from paper_2607_06631_gb300 import dfs, host
+    cfg = synth.tiny()
+    shared, layers, m, acts = synth.make_problem(cfg)
+    prob = host.DeviceProblem(cfg, shared, layers, m, acts)
+    ref_plan = prob.create_plan()
+    ref = torch.empty_like(prob.x)
+    dfs.dfs_block_forward(ref_plan, 2, prob.x, prob.t_emb[2], ref)
+    dfs.dfs_plan_sync(ref_plan)
+    monkeypatch.setenv("DFS_FAULT_LAUNCH", "5")
+    plan = prob.create_plan()
+    monkeypatch.delenv("DFS_FAULT_LAUNCH")
+    out = torch.zeros_like(prob.x)
+    with pytest.raises(dfs.DfsError) as e:
+        dfs.dfs_block_forward(plan, 2, prob.x, prob.t_emb[2], out)
+    assert e.value.status == dfs.DFS_ECUDA and "injected" in str(e.value)
+    dfs.dfs_plan_sync(plan)
+    assert not host.to_bits(out).any()
+    dfs.dfs_block_forward(plan, 2, prob.x, prob.t_emb[2], out)
+    dfs.dfs_plan_sync(plan)
+    np.testing.assert_array_equal(host.to_bits(out), host.to_bits(ref))
+
+
 def test_bounded_wait_reports_timeout_and_context_survives():
     """A wait that nothing completes gives up after about a second, the host reads
     DFS_ETIMEOUT, and the next forward on the same context is correct."""

@@ -103,3 +103,47 @@ def test_wan14b_union_engine_bit_identical_to_compacted():
     # step 0 keeps every unit, so the union is the full layer (4 d^2 + 2 d F bf16 = 493 MB);
     # the compacted engine holds the four steps' copies (1503 MB)
     assert 0.49e9 < mem[1] < 0.50e9 and 1.50e9 < mem[0] < 1.51e9
+
+
+def test_wan14b_x40_stack_sampled_layers_teacher_forced():
+    """The 40-layer Wan-14B-shaped stack with cross-attention (union engine), one pruned
+    denoising step run layer by layer on the GPU; layers 0, 19 and 39 checked against the
+    oracle on sampled rows, each fed the GPU's own output of the layer before it."""
+    import copy
+    import torch
+    from paper_2607_06631_gb300 import build, dfs, host
+    build.build()
+    cfg = copy.deepcopy(synth.wan14b_stack(40))
+    cfg.engine = 1
+    step, pick = 2, (0, 19, 39)
+    layers, w_t, b_t = host.random_device_stack(cfg)
+    masks = synth.make_masks(cfg)
+    acts = synth.make_activations(cfg)
+    x, temb, ctx = host.to_device(acts["x"]), host.to_device(acts["t_emb"]), host.to_device(acts["ctx"])
+    plan = dfs.dfs_plan_create(cfg, layers, w_t, b_t, masks, ctx)
+    host_w = {l: {k: host.to_bits(v) for k, v in layers[l].items()} for l in pick}
+    shared = {"w_t": host.to_bits(w_t), "b_t": host.to_bits(b_t)}
+    del layers, w_t, b_t
+    torch.cuda.empty_cache()
+    rows = sample_rows(cfg.n_tokens, 16, 32)
+    bufs = (torch.empty_like(x), torch.empty_like(x))
+    cur, seen = x, {}
+    for l in range(cfg.n_layers):
+        dst = bufs[l % 2]
+        dfs.dfs_block_forward_layer(plan, step, l, cur, temb[step], dst)
+        if l in pick:
+            dfs.dfs_plan_sync(plan)
+            seen[l] = (host.to_bits(cur), host.to_bits(dst[torch.from_numpy(rows).cuda()]))
+        cur = dst
+    dfs.dfs_plan_sync(plan)
+    plan.close()
+    W = synth.widen(shared)
+    X = synth.widen(acts)
+    for l in pick:
+        x_in, out_rows = seen.pop(l)
+        xin = synth.bits_to_f64(x_in)
+        LW = synth.widen(host_w.pop(l))
+        ref = O.block_forward_compacted(cfg, W, LW, masks, step, l, xin, X["t_emb"][step], X["ctx"], rows=rows)
+        got = synth.bits_to_f64(out_rows)
+        e, b = rel_err(got, ref), branch_err(got, ref, xin[rows])
+        assert e <= TOL and b <= TOL, (l, e, b)
