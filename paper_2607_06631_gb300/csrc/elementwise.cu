@@ -24,6 +24,20 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return warp_sum(t);
 }
 
+// Two sums over the whole CTA in one reduction (one pair of barriers); every thread gets both.
+__device__ __forceinline__ float2 block_sum2(float a, float b, float (*red)[32]) {
+  a = warp_sum(a);
+  b = warp_sum(b);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
+  __syncthreads();
+  if (l == 0) {
+    red[0][w] = a;
+    red[1][w] = b;
+  }
+  __syncthreads();
+  return make_float2(warp_sum(l < nw ? red[0][l] : 0.f), warp_sum(l < nw ? red[1][l] : 0.f));
+}
+
 // ------------------------------------------------------------------ K1 compaction
 
 __global__ void gather_rows_kernel(bf16* __restrict__ dst, long long ld_dst, const bf16* __restrict__ src,
@@ -89,52 +103,60 @@ __global__ void add_table_kernel(float* out, const float* base, const bf16* e, i
 
 // ------------------------------------------------------------------ K2 / K7 row LayerNorm
 
-constexpr int kNormThreads = 256;
-constexpr int kNormMaxVec = 4;  // up to 256 * 4 * 8 = 8192 columns
 
+// One CTA of NT threads per row with the row held in registers (VPT 8-wide vectors per thread;
+// 128 threads and 8 CTAs per SM up to 5120 columns, 256 threads beyond): the row is read from
+// memory once.  Mean and variance come from one
+// CTA reduction of two sums in the shifted-data form: sums of x - K and (x - K)^2 with K the
+// row's first element, which keeps E[(x-K)^2] - E[x-K]^2 free of cancellation however large
+// the row's mean.
 template <bool F32IN>
-__global__ void __launch_bounds__(kNormThreads) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
-                                                                int cols, const float* __restrict__ mul,
-                                                                float mul_bias, const float* __restrict__ add,
-                                                                float eps) {
-  __shared__ float red[32];
-  const long long row = blockIdx.x;
-  const int nvec = cols >> 3;
-  float v[kNormMaxVec][8];
-  float s = 0.f;
-#pragma unroll
-  for (int k = 0; k < kNormMaxVec; ++k) {
-    const int c = threadIdx.x + k * blockDim.x;
-    if (c < nvec) {
-      if (F32IN) {
-        const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(xv) + row * cols) + 2 * c;
-        const float4 a = p[0], b = p[1];
-        v[k][0] = a.x; v[k][1] = a.y; v[k][2] = a.z; v[k][3] = a.w;
-        v[k][4] = b.x; v[k][5] = b.y; v[k][6] = b.z; v[k][7] = b.w;
-      } else {
-        unpack_bf16x8(reinterpret_cast<const uint4*>(static_cast<const bf16*>(xv) + row * cols)[c], v[k]);
-      }
-#pragma unroll
-      for (int i = 0; i < 8; ++i) s += v[k][i];
-    }
+__device__ __forceinline__ void load_vec8(const void* xv, long long off, float (&v)[8]) {
+  if (F32IN) {
+    const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(xv) + off);
+    const float4 a = p[0], b = p[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  } else {
+    unpack_bf16x8(*reinterpret_cast<const uint4*>(static_cast<const bf16*>(xv) + off), v);
   }
-  const float mean = block_sum(s, red) / cols;
-  float q = 0.f;
+}
+
+template <bool F32IN, int VPT, int NT>
+__global__ void __launch_bounds__(NT, 1024 / NT) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
+                                                                   int cols, const float* __restrict__ mul,
+                                                                   float mul_bias, const float* __restrict__ add,
+                                                                   float eps) {
+  __shared__ float red[2][32];
+  const long long r0 = static_cast<long long>(blockIdx.x) * cols;
+  const int nvec = cols >> 3;
+  const float K = F32IN ? static_cast<const float*>(xv)[r0] : bf16_to_f32(static_cast<const bf16*>(xv)[r0]);
+  float v[VPT][8];
 #pragma unroll
-  for (int k = 0; k < kNormMaxVec; ++k) {
-    const int c = threadIdx.x + k * blockDim.x;
+  for (int k = 0; k < VPT; ++k) {
+    const int c = threadIdx.x + k * NT;
+    if (c < nvec) load_vec8<F32IN>(xv, r0 + 8LL * c, v[k]);
+  }
+  float s = 0.f, q = 0.f;
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    const int c = threadIdx.x + k * NT;
     if (c < nvec) {
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const float d = v[k][i] - mean;
-        q += d * d;
+        const float d = v[k][i] - K;
+        s += d;
+        q = fmaf(d, d, q);
       }
     }
   }
-  const float rstd = rsqrtf(block_sum(q, red) / cols + eps);
+  const float2 t = block_sum2(s, q, red);
+  const float ms = t.x / cols;
+  const float mean = K + ms;
+  const float rstd = rsqrtf(fmaxf(t.y / cols - ms * ms, 0.f) + eps);
 #pragma unroll
-  for (int k = 0; k < kNormMaxVec; ++k) {
-    const int c = threadIdx.x + k * blockDim.x;
+  for (int k = 0; k < VPT; ++k) {
+    const int c = threadIdx.x + k * NT;
     if (c < nvec) {
       const float4* m4 = reinterpret_cast<const float4*>(mul) + 2 * c;
       const float4* a4 = reinterpret_cast<const float4*>(add) + 2 * c;
@@ -144,9 +166,34 @@ __global__ void __launch_bounds__(kNormThreads) row_norm_kernel(bf16* __restrict
       float o[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) o[i] = fmaf((v[k][i] - mean) * rstd, mul_bias + mm[i], aa[i]);
-      reinterpret_cast<uint4*>(y + row * cols)[c] = pack_bf16x8(o);
+      *reinterpret_cast<uint4*>(y + r0 + 8LL * c) = pack_bf16x8(o);
     }
   }
+}
+
+template <bool F32IN>
+cudaError_t row_norm_vpt(bf16* y, const void* x, int rows, int cols, const float* mul, float mul_bias,
+                         const float* add, float eps, cudaStream_t s) {
+  const int nvec = cols / 8;
+#define DFS_ROW_NORM(V, N) row_norm_kernel<F32IN, V, N><<<rows, N, 0, s>>>(y, x, cols, mul, mul_bias, add, eps)
+  if (nvec <= 5 * 128) {
+    switch ((nvec + 127) / 128) {
+      case 1: DFS_ROW_NORM(1, 128); break;
+      case 2: DFS_ROW_NORM(2, 128); break;
+      case 3: DFS_ROW_NORM(3, 128); break;
+      case 4: DFS_ROW_NORM(4, 128); break;
+      default: DFS_ROW_NORM(5, 128); break;
+    }
+  } else if (nvec <= 4 * 256) {
+    switch ((nvec + 255) / 256) {
+      case 3: DFS_ROW_NORM(3, 256); break;
+      default: DFS_ROW_NORM(4, 256); break;
+    }
+  } else {
+    return cudaErrorInvalidValue;  // more than 8192 columns
+  }
+#undef DFS_ROW_NORM
+  return cudaGetLastError();
 }
 
 // ------------------------------------------------------------------ K3 QK RMSNorm + RoPE
@@ -167,10 +214,14 @@ struct QkParams {
 };
 
 // One CTA per token row.  The row stays in registers as raw bf16 vectors (VPT 16-byte
-// vectors per thread), so several rows per SM are in flight at once.
+// vectors per thread), so several rows per SM are in flight at once.  The rotation of the
+// row's token (cos, sin per pair of a head, the same for every head) is built once in shared
+// memory from the per-band tables while the row loads, and the q and k statistics share one
+// reduction.
 template <int VPT>
 __global__ void __launch_bounds__(kQkThreads, 4) qk_norm_rope_kernel(const QkParams p) {
-  __shared__ float red[32];
+  __shared__ float red[2][32];
+  __shared__ float rcos[64], rsin[64];
   const long long row = blockIdx.x;
   bf16* base = p.buf + row * p.ld;
   const int nvq = p.nq >> 3, nv = (p.nq + p.nk) >> 3;
@@ -181,9 +232,35 @@ __global__ void __launch_bounds__(kQkThreads, 4) qk_norm_rope_kernel(const QkPar
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
     const int c = threadIdx.x + k * kQkThreads;
+    if (c < nv) raw[k] = reinterpret_cast<const uint4*>(base)[c];
+  }
+  if (p.rope && threadIdx.x < (p.head_dim >> 1)) {
+    const int hw = p.t.grid_h * p.t.grid_w;
+    const int f = static_cast<int>(row / hw);
+    const int rem = static_cast<int>(row - static_cast<long long>(f) * hw);
+    const int yy = rem / p.t.grid_w, xx = rem - yy * p.t.grid_w;
+    const int j = threadIdx.x;
+    float cs, sn;
+    if (j < p.t.p_t) {
+      cs = __ldg(p.t.cos_t + f * p.t.p_t + j);
+      sn = __ldg(p.t.sin_t + f * p.t.p_t + j);
+    } else if (j < p.t.p_t + p.t.p_h) {
+      const int jj = j - p.t.p_t;
+      cs = __ldg(p.t.cos_h + yy * p.t.p_h + jj);
+      sn = __ldg(p.t.sin_h + yy * p.t.p_h + jj);
+    } else {
+      const int jj = j - p.t.p_t - p.t.p_h;
+      cs = __ldg(p.t.cos_w + xx * p.t.p_w + jj);
+      sn = __ldg(p.t.sin_w + xx * p.t.p_w + jj);
+    }
+    rcos[j] = cs;
+    rsin[j] = sn;
+  }
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    const int c = threadIdx.x + k * kQkThreads;
     float ss = 0.f;
     if (c < nv) {
-      raw[k] = reinterpret_cast<const uint4*>(base)[c];
       float v[8];
       unpack_bf16x8(raw[k], v);
 #pragma unroll
@@ -194,10 +271,9 @@ __global__ void __launch_bounds__(kQkThreads, 4) qk_norm_rope_kernel(const QkPar
   }
   float rq = 0.f, rk = 0.f;
   if (p.mode == 0) {
-    const float tq = block_sum(sq, red);
-    const float tk = block_sum(sk, red);
-    rq = p.nq > 0 ? rsqrtf(tq / p.nq + p.eps) : 0.f;
-    rk = p.nk > 0 ? rsqrtf(tk / p.nk + p.eps) : 0.f;
+    const float2 t = block_sum2(sq, sk, red);  // its barriers also publish the rotation table
+    rq = p.nq > 0 ? rsqrtf(t.x / p.nq + p.eps) : 0.f;
+    rk = p.nk > 0 ? rsqrtf(t.y / p.nk + p.eps) : 0.f;
   } else {
     // per head: the vph threads holding one head are consecutive lanes of one warp
 #pragma unroll
@@ -206,14 +282,7 @@ __global__ void __launch_bounds__(kQkThreads, 4) qk_norm_rope_kernel(const QkPar
       for (int o = vph >> 1; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
       hs[k] = rsqrtf(t / p.head_dim + p.eps);
     }
-  }
-  int f = 0, yy = 0, xx = 0;
-  if (p.rope) {
-    const int hw = p.t.grid_h * p.t.grid_w;
-    f = static_cast<int>(row / hw);
-    const int rem = static_cast<int>(row - static_cast<long long>(f) * hw);
-    yy = rem / p.t.grid_w;
-    xx = rem - yy * p.t.grid_w;
+    if (p.rope) __syncthreads();
   }
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
@@ -231,20 +300,7 @@ __global__ void __launch_bounds__(kQkThreads, 4) qk_norm_rope_kernel(const QkPar
         const int j0 = (ch0 % p.head_dim) >> 1;  // first rotation pair of this vector
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          const int j = j0 + i;
-          float cs, sn;
-          if (j < p.t.p_t) {
-            cs = __ldg(p.t.cos_t + f * p.t.p_t + j);
-            sn = __ldg(p.t.sin_t + f * p.t.p_t + j);
-          } else if (j < p.t.p_t + p.t.p_h) {
-            const int jj = j - p.t.p_t;
-            cs = __ldg(p.t.cos_h + yy * p.t.p_h + jj);
-            sn = __ldg(p.t.sin_h + yy * p.t.p_h + jj);
-          } else {
-            const int jj = j - p.t.p_t - p.t.p_h;
-            cs = __ldg(p.t.cos_w + xx * p.t.p_w + jj);
-            sn = __ldg(p.t.sin_w + xx * p.t.p_w + jj);
-          }
+          const float cs = rcos[j0 + i], sn = rsin[j0 + i];
           const float a = o[2 * i], b = o[2 * i + 1];
           o[2 * i] = a * cs - b * sn;
           o[2 * i + 1] = a * sn + b * cs;
@@ -335,14 +391,9 @@ cudaError_t launch_add_table(float* out, const float* base, const bf16* e, int n
 cudaError_t launch_row_norm(bf16* y, const void* x, int x_f32, int rows, int cols, const float* mul,
                             float mul_bias, const float* add, float eps, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  if (cols % 8 != 0 || cols > kNormThreads * kNormMaxVec * 8) return cudaErrorInvalidValue;
-  int threads = ((cols / 8 + 31) / 32) * 32;
-  if (threads > kNormThreads) threads = kNormThreads;
-  if (x_f32)
-    row_norm_kernel<true><<<rows, threads, 0, s>>>(y, x, cols, mul, mul_bias, add, eps);
-  else
-    row_norm_kernel<false><<<rows, threads, 0, s>>>(y, x, cols, mul, mul_bias, add, eps);
-  return cudaGetLastError();
+  if (cols % 8 != 0 || cols <= 0) return cudaErrorInvalidValue;
+  return x_f32 ? row_norm_vpt<true>(y, x, rows, cols, mul, mul_bias, add, eps, s)
+               : row_norm_vpt<false>(y, x, rows, cols, mul, mul_bias, add, eps, s);
 }
 
 cudaError_t launch_qk_norm_rope(bf16* buf, long long ld, int rows, int nq, int nk, const bf16* gamma_q,
@@ -355,11 +406,17 @@ cudaError_t launch_qk_norm_rope(bf16* buf, long long ld, int rows, int nq, int n
   p.head_dim = head_dim; p.mode = mode; p.eps = eps;
   p.rope = rope != nullptr;
   if (rope) p.t = *rope; else memset(&p.t, 0, sizeof(p.t));
+  if (head_dim > 128) return cudaErrorInvalidValue;  // the rotation table holds 64 pairs
   const int vpt = ((nq + nk) / 8 + kQkThreads - 1) / kQkThreads;
-  if (vpt <= 1) qk_norm_rope_kernel<1><<<rows, kQkThreads, 0, s>>>(p);
-  else if (vpt <= 2) qk_norm_rope_kernel<2><<<rows, kQkThreads, 0, s>>>(p);
-  else if (vpt <= 4) qk_norm_rope_kernel<4><<<rows, kQkThreads, 0, s>>>(p);
-  else qk_norm_rope_kernel<8><<<rows, kQkThreads, 0, s>>>(p);
+  switch (vpt) {
+    case 1: qk_norm_rope_kernel<1><<<rows, kQkThreads, 0, s>>>(p); break;
+    case 2: qk_norm_rope_kernel<2><<<rows, kQkThreads, 0, s>>>(p); break;
+    case 3: qk_norm_rope_kernel<3><<<rows, kQkThreads, 0, s>>>(p); break;
+    case 4: qk_norm_rope_kernel<4><<<rows, kQkThreads, 0, s>>>(p); break;
+    case 5: qk_norm_rope_kernel<5><<<rows, kQkThreads, 0, s>>>(p); break;
+    case 6: qk_norm_rope_kernel<6><<<rows, kQkThreads, 0, s>>>(p); break;
+    default: qk_norm_rope_kernel<8><<<rows, kQkThreads, 0, s>>>(p); break;
+  }
   return cudaGetLastError();
 }
 

@@ -75,6 +75,14 @@ def test_head_dim_128_tiny():
     check_block(cfg, r0, res)
 
 
+def test_wide_rows_above_5120_channels():
+    """dim 6144 (48 heads x 128): the LayerNorm's 256-thread row layout, 1536-channel q / k rows."""
+    cfg = _custom(dim=6144, n_heads=48, head_dim=128, ffn=2048, heads=(48, 12, 30, 1), chunks=(256, 40, 128, 9),
+                  grid=(2, 4, 5))
+    r0, res = run_block(cfg)
+    check_block(cfg, r0, res)
+
+
 def test_empty_masks_and_block_gate():
     cfg = synth.tiny()
     m = synth.make_masks(cfg)
