@@ -326,6 +326,7 @@ def run_ours(args):
     peaks, peak_src = load_peaks()
     cfg = get_config(args.config, args.grid)
     cfg.engine = dfs.ENGINES[args.engine]
+    cfg.qk_norm_mode = args.qk_norm_mode
     T, L = cfg.n_steps, cfg.n_layers
     stream = torch.cuda.current_stream()
     # the dense reference of the speedups: step 0 when it keeps every unit, else a separate
@@ -528,7 +529,7 @@ def run_ours(args):
             "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": workload_desc(cfg),
-                       "engine": args.engine,
+                       "engine": args.engine, "qk_norm_mode": args.qk_norm_mode,
                        "plan_weight_gb": round(weight_bytes / 1e9, 3),
                        "plan_device_gb": round(device_bytes / 1e9, 3),
                        "l2": "inputs larger than L2 (x %.0f MB, per-step weights read %.0f-%.0f MB); no flush "
@@ -568,6 +569,8 @@ def main():
                          "wan13b_policy (30-layer 4-step denoise, policy-shaped masks), wan13b_model (the same "
                          "layers inside the Wan-shaped model on a latent video), tiny")
     ap.add_argument("--grid", default=None, help="override the latent grid T,H,W (smaller profiling cases)")
+    ap.add_argument("--qk-norm-mode", type=int, choices=(0, 1), default=0,
+                    help="QK RMSNorm over the retained channels of a row (0, default) or per head (1)")
     ap.add_argument("--engine", choices=("compacted", "union"), default="compacted",
                     help="weights per (step, layer) compacted once (default), or one union super-model per "
                          "layer gathered by the projections' TMA producers (Sec. 4.3)")

@@ -83,6 +83,23 @@ def test_wide_rows_above_5120_channels():
     check_block(cfg, r0, res)
 
 
+@pytest.mark.parametrize("case", ["dh128", "ragged", "cross"])
+def test_per_head_qk_norm(case):
+    """qk_norm_mode 1 (QK RMSNorm per head) with head_dim 128, ragged token counts and
+    cross-attention: q, k after RMSNorm + RoPE and the block output against the oracle."""
+    if case == "dh128":
+        cfg = _custom(dim=512, n_heads=4, head_dim=128, ffn=1024, heads=(4, 3, 2, 1), chunks=(128, 100, 50, 16),
+                      grid=(2, 8, 20))
+    elif case == "ragged":
+        cfg = _custom(grid=(3, 10, 13))
+    else:
+        cfg = synth.tiny(has_cross=1)
+    cfg.qk_norm_mode = 1
+    cfg.name += "_mode1"
+    r0, res = run_block(cfg)
+    check_block(cfg, r0, res)
+
+
 def test_empty_masks_and_block_gate():
     cfg = synth.tiny()
     m = synth.make_masks(cfg)

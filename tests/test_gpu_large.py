@@ -61,6 +61,16 @@ def test_wan14b_block_every_step():
         assert e <= TOL and b <= TOL, (s, e, b)
 
 
+def test_wan14b_block_per_head_qk_norm():
+    """qk_norm_mode 1 (QK RMSNorm per head) at full size."""
+    cfg = synth.wan14b()
+    cfg.qk_norm_mode = 1
+    cfg.name = "wan14b_mode1"
+    errs = run_large(cfg, (0, 3), edge=32, spread=64)
+    for s, (e, b) in errs.items():
+        assert e <= TOL and b <= TOL, (s, e, b)
+
+
 def test_wan14b_block_with_cross_attention():
     errs = run_large(synth.wan14b_cross(), (0, 3), edge=32, spread=64)
     for s, (e, b) in errs.items():
