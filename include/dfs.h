@@ -10,7 +10,7 @@
  *     pointers are ordinary CPU memory.  Nothing here takes or returns torch types.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).  All GPU
  *     work is enqueued on it; no entry point synchronises except dfs_plan_create,
- *     dfs_plan_sync and the *_host variants, which say so.
+ *     dfs_plan_sync and dfs_block_forward_host, which say so.
  *   - Errors are returned as dfs_status and never thrown across the ABI; dfs_last_error()
  *     gives a message for the calling thread.  On any error nothing is written to `out`.
  *   - A plan may be used from one host thread at a time.
@@ -129,6 +129,24 @@ dfs_status dfs_block_forward_layer(dfs_plan* plan, int step, int layer, const vo
 dfs_status dfs_block_forward_host(dfs_plan* plan, int step, int layer, const void* x_host,
                                   const void* t_emb_host, void* out_host, void* stream);
 
+/* Asynchronous variant of dfs_block_forward_host for streaming many host-resident inputs:
+ * enqueues the copy of x and t_emb into one of two plan-owned staging slots (on a copy
+ * stream of the plan), the forward (on `stream`) and the copy of the result to `out_host`
+ * (on a second copy stream), and returns without waiting.  Successive calls alternate the
+ * slots, so the input copy of call i+1 and the output copy of call i-1 overlap the forward
+ * of call i.  Ordering and ownership:
+ *   - out_host holds the result once dfs_plan_sync(plan, stream) has returned (it waits for
+ *     the copies of every earlier asynchronous call); until then x_host, t_emb_host and
+ *     out_host are in use by the library: the caller must not write x_host / t_emb_host or
+ *     read out_host (an out_host of an unsynchronised call is not yet a valid x_host).
+ *   - Use one stream for a sequence of calls, as for every forward of a plan.
+ *   - The first call allocates the second slot (2 N dim + dim bf16) and creates two streams
+ *     and six events, all freed by dfs_plan_destroy.  Pinned host memory (cudaHostAlloc)
+ *     is needed for the copies to run asynchronously at full speed.
+ * Errors: as dfs_block_forward_layer, plus DFS_ENOMEM on the first call. */
+dfs_status dfs_block_forward_host_async(dfs_plan* plan, int step, int layer, const void* x_host,
+                                        const void* t_emb_host, void* out_host, void* stream);
+
 /* Allocation-free variant of dfs_block_forward_layer (the paper has no counterpart;
  * this is a deployment convenience).  Same arguments, same kernels, same result; the
  * per-call activation workspace lives in a 16 MiB device array that the library
@@ -238,9 +256,10 @@ dfs_status dfs_plan_flops(const dfs_plan* plan, int step, int layer, double* flo
 dfs_status dfs_plan_workspace(const dfs_plan* plan, int which, void** dev, int64_t* rows,
                               int64_t* cols, int64_t* ld, int* dtype);
 
-/* Waits for `stream` and reports whether any kernel of this plan hit its bounded wait
- * limit since the last call (DFS_ETIMEOUT) or a CUDA error occurred (DFS_ECUDA).
- * Clears the plan's device error word. */
+/* Waits for `stream` (and for the copies of earlier dfs_block_forward_host_async calls)
+ * and reports whether any kernel of this plan hit its bounded wait limit since the last
+ * call (DFS_ETIMEOUT) or a CUDA error occurred (DFS_ECUDA).  Clears the plan's device
+ * error word. */
 dfs_status dfs_plan_sync(dfs_plan* plan, void* stream);
 
 /* Failure-path self test: launches one small kernel on `stream` that waits on a barrier

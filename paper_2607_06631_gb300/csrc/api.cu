@@ -152,6 +152,20 @@ struct dfs_plan {
   bf16* stage_x = nullptr;
   bf16* stage_out = nullptr;
   bf16* stage_t = nullptr;
+  // Two-slot staging ring of dfs_block_forward_host_async (slot 0 is stage_x / stage_out /
+  // stage_t): host->device copies on `h2d`, device->host copies on `d2h`, ordered against
+  // the caller's stream by per-slot events.
+  struct HostRing {
+    bool ready = false;
+    int next = 0;
+    bf16* x[2] = {nullptr, nullptr};
+    bf16* out[2] = {nullptr, nullptr};
+    bf16* t[2] = {nullptr, nullptr};
+    cudaStream_t h2d = nullptr, d2h = nullptr;
+    cudaEvent_t loaded[2] = {nullptr, nullptr};    // slot's inputs on the device
+    cudaEvent_t computed[2] = {nullptr, nullptr};  // slot's forward done (inputs free, output ready)
+    cudaEvent_t drained[2] = {nullptr, nullptr};   // slot's output copied to the host
+  } ring;
   int* err = nullptr;
   std::vector<void*> allocs;
   int last_step = -1, last_layer = -1;
@@ -216,6 +230,16 @@ dfs_status alloc_temp(dfs_plan* P, bf16** out, long long n) {
 void free_plan(dfs_plan* P) {
   if (!P) return;
   for (cudaEvent_t e : P->ev) cudaEventDestroy(e);
+  {
+    dfs_plan::HostRing& R = P->ring;
+    if (R.h2d) cudaStreamSynchronize(R.h2d);
+    if (R.d2h) cudaStreamSynchronize(R.d2h);
+    for (int b = 0; b < 2; ++b)
+      for (cudaEvent_t e : {R.loaded[b], R.computed[b], R.drained[b]})
+        if (e) cudaEventDestroy(e);
+    if (R.h2d) cudaStreamDestroy(R.h2d);
+    if (R.d2h) cudaStreamDestroy(R.d2h);
+  }
   for (void* p : P->allocs) cudaFree(p);
   for (void* p : P->temps) cudaFree(p);
   delete P;
@@ -925,11 +949,76 @@ dfs_status dfs_block_forward(dfs_plan* plan, int step, const void* x, const void
   return dfs_block_forward_layer(plan, step, 0, x, t_emb, out, stream);
 }
 
+namespace {
+
+// Makes `st` wait for every copy the staging ring has in flight.
+dfs_status ring_join(dfs_plan* P, cudaStream_t st) {
+  dfs_plan::HostRing& R = P->ring;
+  if (!R.ready) return DFS_OK;
+  for (int b = 0; b < 2; ++b) {
+    DFS_CK(cudaStreamWaitEvent(st, R.loaded[b], 0));
+    DFS_CK(cudaStreamWaitEvent(st, R.drained[b], 0));
+  }
+  return DFS_OK;
+}
+
+// First use of the ring: the second slot's device buffers, two copy streams, six events.
+dfs_status ring_init(dfs_plan* P) {
+  dfs_plan::HostRing& R = P->ring;
+  if (R.ready) return DFS_OK;
+  const long long n = P->N * P->cfg.dim;
+  R.x[0] = P->stage_x;
+  R.out[0] = P->stage_out;
+  R.t[0] = P->stage_t;
+  dfs_status e;
+  if (!R.x[1] && ((e = alloc_n(P, &R.x[1], n)) || (e = alloc_n(P, &R.out[1], n)) ||
+                  (e = alloc_n(P, &R.t[1], P->cfg.dim))))
+    return e;
+  if (!R.h2d) DFS_CK(cudaStreamCreateWithFlags(&R.h2d, cudaStreamNonBlocking));
+  if (!R.d2h) DFS_CK(cudaStreamCreateWithFlags(&R.d2h, cudaStreamNonBlocking));
+  for (int b = 0; b < 2; ++b)
+    for (cudaEvent_t* ev : {&R.loaded[b], &R.computed[b], &R.drained[b]})
+      if (!*ev) DFS_CK(cudaEventCreateWithFlags(ev, cudaEventDisableTiming));
+  R.ready = true;
+  return DFS_OK;
+}
+
+}  // namespace
+
+dfs_status dfs_block_forward_host_async(dfs_plan* plan, int step, int layer, const void* x_host,
+                                        const void* t_emb_host, void* out_host, void* stream) {
+  dfs_status e = check_forward_args(plan, step, layer, x_host, t_emb_host, out_host);
+  if (e) return e;
+  if ((e = ring_init(plan))) return e;
+  dfs_plan::HostRing& R = plan->ring;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int b = R.next;
+  const size_t bytes = sizeof(bf16) * plan->N * plan->cfg.dim;
+  // inputs: into slot b once the forward two calls back has finished reading it
+  DFS_CK(cudaStreamWaitEvent(R.h2d, R.computed[b], 0));
+  DFS_CK(cudaMemcpyAsync(R.x[b], x_host, bytes, cudaMemcpyHostToDevice, R.h2d));
+  DFS_CK(cudaMemcpyAsync(R.t[b], t_emb_host, sizeof(bf16) * plan->cfg.dim, cudaMemcpyHostToDevice, R.h2d));
+  DFS_CK(cudaEventRecord(R.loaded[b], R.h2d));
+  // forward on the caller's stream once the inputs are in and slot b's last output is out
+  DFS_CK(cudaStreamWaitEvent(st, R.loaded[b], 0));
+  DFS_CK(cudaStreamWaitEvent(st, R.drained[b], 0));
+  if ((e = block_layer(plan, step, layer, R.x[b], R.t[b], R.out[b], st))) return e;
+  DFS_CK(cudaEventRecord(R.computed[b], st));
+  // output: back to the host while the caller's stream moves on
+  DFS_CK(cudaStreamWaitEvent(R.d2h, R.computed[b], 0));
+  DFS_CK(cudaMemcpyAsync(out_host, R.out[b], bytes, cudaMemcpyDeviceToHost, R.d2h));
+  DFS_CK(cudaEventRecord(R.drained[b], R.d2h));
+  R.next = b ^ 1;
+  return DFS_OK;
+}
+
 dfs_status dfs_block_forward_host(dfs_plan* plan, int step, int layer, const void* x_host, const void* t_emb_host,
                                   void* out_host, void* stream) {
   dfs_status e = check_forward_args(plan, step, layer, x_host, t_emb_host, out_host);
   if (e) return e;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // slot 0 of the asynchronous ring may still be in use by earlier asynchronous calls
+  if ((e = ring_join(plan, st))) return e;
   const size_t bytes = sizeof(bf16) * plan->N * plan->cfg.dim;
   DFS_CK(cudaMemcpyAsync(plan->stage_x, x_host, bytes, cudaMemcpyHostToDevice, st));
   DFS_CK(cudaMemcpyAsync(plan->stage_t, t_emb_host, sizeof(bf16) * plan->cfg.dim, cudaMemcpyHostToDevice, st));
@@ -1158,6 +1247,8 @@ dfs_status dfs_plan_workspace(const dfs_plan* P, int which, void** dev, int64_t*
 dfs_status dfs_plan_sync(dfs_plan* P, void* stream) {
   if (!P) return fail(DFS_EINVAL, "plan is NULL");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  dfs_status e = ring_join(P, st);
+  if (e) return e;
   DFS_CK(cudaStreamSynchronize(st));
   int herr = 0;
   DFS_CK(cudaMemcpy(&herr, P->err, sizeof(int), cudaMemcpyDeviceToHost));

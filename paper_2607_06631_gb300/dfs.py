@@ -21,7 +21,7 @@ _STATUS = {0: "DFS_OK", 1: "DFS_EINVAL", 2: "DFS_ENOMEM", 3: "DFS_ECUDA", 4: "DF
            5: "DFS_EUNSUPPORTED"}
 
 EXPORTED = ("dfs_plan_create", "dfs_block_forward", "dfs_block_forward_layer", "dfs_block_forward_host",
-            "dfs_block_forward_noalloc",
+            "dfs_block_forward_host_async", "dfs_block_forward_noalloc",
             "dfs_denoise", "dfs_plan_indices", "dfs_plan_panel", "dfs_plan_union_panel", "dfs_plan_memory",
             "dfs_plan_flops", "dfs_plan_workspace",
             "dfs_plan_sync", "dfs_selftest_wait_timeout", "dfs_plan_profile", "dfs_plan_profile_read", "dfs_gates_from_soft_masks",
@@ -92,6 +92,7 @@ def lib() -> ctypes.CDLL:
         L.dfs_block_forward.argtypes = [vp, i32, vp, vp, vp, vp]
         L.dfs_block_forward_layer.argtypes = [vp, i32, i32, vp, vp, vp, vp]
         L.dfs_block_forward_host.argtypes = [vp, i32, i32, vp, vp, vp, vp]
+        L.dfs_block_forward_host_async.argtypes = [vp, i32, i32, vp, vp, vp, vp]
         L.dfs_block_forward_noalloc.argtypes = [vp, i32, i32, vp, vp, vp, vp]
         L.dfs_denoise.argtypes = [vp, vp, i32, vp, vp]
         L.dfs_plan_indices.argtypes = [vp, i32, i32, i32, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(i32)]
@@ -234,6 +235,12 @@ def dfs_block_forward_layer(plan, step: int, layer: int, x, t_emb, out, stream=N
 def dfs_block_forward_host(plan, step: int, layer: int, x_host, t_emb_host, out_host, stream=None):
     _check(lib().dfs_block_forward_host(_h(plan), step, layer, _ptr(x_host), _ptr(t_emb_host),
                                         _ptr(out_host), _stream(stream)))
+
+
+def dfs_block_forward_host_async(plan, step: int, layer: int, x_host, t_emb_host, out_host, stream=None):
+    """Enqueue-only host-buffer forward; out_host is valid after dfs_plan_sync(plan, stream)."""
+    _check(lib().dfs_block_forward_host_async(_h(plan), step, layer, _ptr(x_host), _ptr(t_emb_host),
+                                              _ptr(out_host), _stream(stream)))
 
 
 def dfs_block_forward_noalloc(plan, step: int, layer: int, x, t_emb, out, stream=None):

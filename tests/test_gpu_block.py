@@ -135,6 +135,37 @@ def test_host_buffers_match_device_buffers():
     np.testing.assert_array_equal(host.to_bits(o_h), host.to_bits(out))
 
 
+def test_async_host_ring_matches_device_buffers():
+    """Five asynchronous host-buffer forwards (both staging slots reused, a synchronous call
+    in between) give each call's own device-path result."""
+    import torch
+    from paper_2607_06631_gb300 import dfs, host
+    cfg = synth.tiny()
+    r0, _ = run_block(cfg, steps=[], want_intermediates=False)
+    plan, prob = r0["plan"], r0["prob"]
+    g = torch.Generator().manual_seed(7)
+    xs = [(prob.x.float().cpu() + 0.1 * k * torch.randn(prob.x.shape, generator=g)).to(prob.x.dtype)
+          for k in range(6)]
+    steps = [0, 3, 1, 2, 0, 3]
+    want = []
+    for k, s in enumerate(steps):
+        out = torch.empty_like(prob.x)
+        dfs.dfs_block_forward(plan, s, xs[k].cuda(), prob.t_emb[s], out)
+        want.append(out)
+    dfs.dfs_plan_sync(plan)
+    x_h = [x.pin_memory() for x in xs]
+    t_h = [prob.t_emb[s].cpu().pin_memory() for s in steps]
+    o_h = [torch.empty_like(x_h[0]).pin_memory() for _ in steps]
+    for k in range(3):
+        dfs.dfs_block_forward_host_async(plan, steps[k], 0, x_h[k], t_h[k], o_h[k])
+    dfs.dfs_block_forward_host(plan, steps[3], 0, x_h[3], t_h[3], o_h[3])
+    for k in range(4, 6):
+        dfs.dfs_block_forward_host_async(plan, steps[k], 0, x_h[k], t_h[k], o_h[k])
+    dfs.dfs_plan_sync(plan)
+    for k in range(len(steps)):
+        np.testing.assert_array_equal(host.to_bits(o_h[k]), host.to_bits(want[k]), err_msg=f"call {k}")
+
+
 def test_denoise_small_stack():
     import torch
     from paper_2607_06631_gb300 import dfs, host
