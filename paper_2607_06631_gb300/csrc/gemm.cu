@@ -156,6 +156,89 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int row, int c
   }
 }
 
+// Raw 16-byte words of one 32-column chunk of this thread's residual row (fp32: 8 words,
+// bf16: the first 4).
+__device__ __forceinline__ void load_res_chunk(int res_f32, const char* rrow, int c, uint4 (&w)[8]) {
+  if (res_f32) {
+    const uint4* src = reinterpret_cast<const uint4*>(rrow + c * 128);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) w[q] = src[q];
+  } else {
+    const uint4* src = reinterpret_cast<const uint4*>(rrow + c * 64);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) w[q] = src[q];
+  }
+}
+
+// kEpiGatedRes over one full row of a 256-column tile (row < M, all columns < N): the same
+// arithmetic as epilogue_chunk, with the residual loads of chunk c + 2 issued before chunk c
+// is processed, so that each warp keeps three chunks of loads in flight instead of waiting
+// out one memory latency per 32 columns.  The residual may be the output itself (in-place
+// update): every element is still read by its own thread before that thread writes it.
+__device__ __forceinline__ void epilogue_gated_row(const GemmArgs& p, int row, int colb, uint32_t taddr) {
+  const char* rrow = static_cast<const char*>(p.res) +
+                     (static_cast<long long>(row) * p.ldr + colb) * (p.res_f32 ? 4 : 2);
+  uint4 w[3][8];
+  load_res_chunk(p.res_f32, rrow, 0, w[0]);
+  load_res_chunk(p.res_f32, rrow, 1, w[1]);
+#pragma unroll
+  for (int c = 0; c < kGemmBN / 32; ++c) {
+    if (c + 2 < kGemmBN / 32) load_res_chunk(p.res_f32, rrow, c + 2, w[(c + 2) % 3]);
+    const int col0 = colb + 32 * c;
+    float v[32];
+    tmem_ld32(taddr + 32 * c, v);
+    if (p.bias != nullptr) {
+      const uint4* b4 = reinterpret_cast<const uint4*>(p.bias + col0);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float f[8];
+        unpack_bf16x8(__ldg(b4 + q), f);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[8 * q + i] += f[i];
+      }
+    }
+    float g[32];
+    if (p.gate != nullptr) {
+      const float4* g4 = reinterpret_cast<const float4*>(p.gate + col0);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float4 t = __ldg(g4 + q);
+        g[4 * q] = t.x; g[4 * q + 1] = t.y; g[4 * q + 2] = t.z; g[4 * q + 3] = t.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) g[j] = 1.f;
+    }
+    float r[32];
+    const uint4(&wc)[8] = w[c % 3];
+    if (p.res_f32) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        r[4 * q] = __uint_as_float(wc[q].x); r[4 * q + 1] = __uint_as_float(wc[q].y);
+        r[4 * q + 2] = __uint_as_float(wc[q].z); r[4 * q + 3] = __uint_as_float(wc[q].w);
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float f[8];
+        unpack_bf16x8(wc[q], f);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) r[8 * q + i] = f[i];
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = fmaf(g[j], v[j], r[j]);
+    if (p.out_f32) {
+      float* op = static_cast<float*>(p.out) + static_cast<long long>(row) * p.ldo + col0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        *reinterpret_cast<float4*>(op + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+    } else {
+      store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, 32);
+    }
+  }
+}
+
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_bf16_tcgen05(const __grid_constant__ GemmArgs p) {
   extern __shared__ uint8_t smem_raw[];
@@ -290,17 +373,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
         tc_fence_after();
       }
-      for (int c = 0; c < kGemmBN; c += 32) {
-        const int col0 = nt * kGemmBN + c;
-        if (col0 >= p.N) break;
-        float v[32];
-        if (kb > 0) {
-          tmem_ld32(tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * kGemmBN + c, v);
-        } else {
+      const uint32_t tacc = tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * kGemmBN;
+      // warp-uniform choice: the TMEM loads on both paths are warp-collective
+      if (p.mode == kEpiGatedRes && kb > 0 && (nt + 1) * kGemmBN <= p.N && __all_sync(0xffffffffu, row < p.M)) {
+        epilogue_gated_row(p, row, nt * kGemmBN, tacc);
+      } else {
+        for (int c = 0; c < kGemmBN; c += 32) {
+          const int col0 = nt * kGemmBN + c;
+          if (col0 >= p.N) break;
+          float v[32];
+          if (kb > 0) {
+            tmem_ld32(tacc + c, v);
+          } else {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = 0.f;
+            for (int j = 0; j < 32; ++j) v[j] = 0.f;
+          }
+          epilogue_chunk(p, row, col0, v);
         }
-        epilogue_chunk(p, row, col0, v);
       }
       if (kb > 0) {
         // this accumulator is read out: one arrival per warp on the even CTA's barrier
