@@ -32,14 +32,18 @@ def branch_err(out, ref, x) -> float:
     return float(extra.max() / den) if den > 0 else float(extra.max())
 
 
-def run_block(cfg, seed_tag="", masks=None, steps=None, layer=0, want_intermediates=True, rows=None):
+def run_block(cfg, seed_tag="", masks=None, steps=None, layer=0, want_intermediates=True, rows=None,
+              patch=None):
     """Runs every requested step of `layer` on the GPU and the oracle (compacted mode).
+    `patch(layers)`, if given, edits the seeded bf16 layer weights in place first.
 
     Returns a list of dicts with the GPU output, the oracle output and intermediates."""
     import torch
     from paper_2607_06631_gb300 import dfs, host
 
     shared, layers, m, acts = synth.make_problem(cfg, seed_tag)
+    if patch is not None:
+        patch(layers)
     if masks is not None:
         m = masks
     prob = host.DeviceProblem(cfg, shared, layers, m, acts)

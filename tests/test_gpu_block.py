@@ -75,6 +75,52 @@ def test_head_dim_128_tiny():
     check_block(cfg, r0, res)
 
 
+@pytest.mark.parametrize("head_dim,gamma", [(64, 4.0), (128, 4.0), (64, 8.0)])
+def test_peaky_scores_rescale_the_running_max(head_dim, gamma):
+    """q / k norm scales multiplied by gamma make the scores gamma^2 times larger, so that in
+    many rows a later key block raises the row max by more than 2^8 (log2 units): the kernel
+    then rescales the row's O accumulator and sum (with the default scales that never happens
+    at these sizes).  The attention output is compared with the plain softmax of the GPU's
+    own bf16 q, k and V (the attention kernel alone; upstream bf16 rounding of q and k moves
+    such peaky scores by more than the block tolerance), and, at gamma 4, the block output
+    with the oracle at a tolerance that allows for that rounding (630 tokens: a ragged
+    last key block)."""
+    if head_dim == 64:
+        cfg = _custom(grid=(2, 15, 21))
+    else:
+        cfg = _custom(dim=512, n_heads=4, head_dim=128, ffn=1024, heads=(4, 3, 2, 1), chunks=(128, 100, 50, 16),
+                      grid=(2, 15, 21))
+
+    def scale_gammas(layers):
+        for lw in layers:
+            for k in ("gq", "gk"):
+                lw[k] = synth.f32_to_bf16_bits(synth.bits_to_f32(lw[k]) * gamma)
+
+    r0, res = run_block(cfg, steps=[0, 2], patch=scale_gammas)
+    dh = cfg.head_dim
+    sl2 = np.log2(np.e) / np.sqrt(dh)
+    moves = 0
+    for r in res:
+        N = r["ws_qk"].shape[0]
+        hd = r["ws_qk"].shape[1] // 2
+        q = r["ws_qk"][:, :hd].reshape(N, -1, dh)
+        k = r["ws_qk"][:, hd:].reshape(N, -1, dh)
+        v = r["ws_vt"].T.reshape(N, -1, dh)
+        want = O.attention(q, k, v).reshape(N, hd)
+        assert rel_err(r["ws_attn"], want) <= 1e-2, ("attn vs softmax of the GPU's q, k, v", r["step"],
+                                                      rel_err(r["ws_attn"], want))
+        for h in range(q.shape[1]):
+            S = (q[:, h] @ k[:, h].T) * sl2
+            m_run = S[:, :128].max(1)
+            for j in range(1, (N + 127) // 128):
+                mx = S[:, 128 * j:128 * (j + 1)].max(1)
+                moves += int((mx > m_run + 8).sum())
+                m_run = np.where(mx > m_run + 8, mx, m_run)
+        if gamma <= 4:
+            assert branch_err(r["out"], r["ref"], r0["x"]) <= 0.1, ("out - x", r["step"])
+    assert moves > 100, moves
+
+
 def test_wide_rows_above_5120_channels():
     """dim 6144 (48 heads x 128): the LayerNorm's 256-thread row layout, 1536-channel q / k rows."""
     cfg = _custom(dim=6144, n_heads=48, head_dim=128, ffn=2048, heads=(48, 12, 30, 1), chunks=(256, 40, 128, 9),
