@@ -14,6 +14,13 @@
  *   - Errors are returned as dfs_status and never thrown across the ABI; dfs_last_error()
  *     gives a message for the calling thread.  On any error nothing is written to `out`.
  *   - A plan may be used from one host thread at a time.
+ *   - CUDA graphs: dfs_block_forward, dfs_block_forward_layer, dfs_block_forward_noalloc
+ *     (after its first call on the device), dfs_denoise, dfs_model_forward and
+ *     dfs_model_denoise enqueue only kernel launches and device-to-device copies, with no
+ *     allocation and no synchronisation, so a call made while `stream` is capturing
+ *     (cudaStreamBeginCapture) is recorded into the graph.  A replay reuses the pointers
+ *     and host scalars (timesteps) of the capture and reads the device buffers' contents at
+ *     replay time.  Per-kernel profiling (dfs_plan_profile) must be off while capturing.
  */
 #ifndef DFS_H_
 #define DFS_H_
