@@ -267,12 +267,20 @@ CPU_ROWS = 32
 
 
 def cpu_baseline(cfg):
+    import oracle as O
     prob = load_problem_f64(cfg)
     step = cfg.n_steps - 1
     dt, fl = oracle_sample(cfg, prob, step, CPU_ROWS)
+    # the whole block of that step at the sample's FLOP rate (an extrapolation, not a run)
+    h_s, f_s = cfg.heads_kept[step][0], 8 * cfg.chunks_kept[step][0]
+    hc = cfg.xheads_kept[step][0] if cfg.has_cross else 0
+    full = O.block_flops(cfg.n_tokens, cfg.dim, cfg.head_dim, h_s, f_s, hc, cfg.ctx_len)
     return {"value": fl / dt / 1e12, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
             "sample": "float64 oracle, MoM step %d, %d query rows (keys/values over all %d tokens): "
-                      "%.3e counted FLOPs in %.1f s" % (step, CPU_ROWS, cfg.n_tokens, fl, dt)}
+                      "%.3e counted FLOPs in %.1f s" % (step, CPU_ROWS, cfg.n_tokens, fl, dt),
+            "block_seconds_extrapolated": round(full / (fl / dt), 2),
+            "extrapolation": "one full block of MoM step %d (%.3e algorithmic FLOPs) at the sample's FLOP rate"
+                             % (step, full)}
 
 
 def run_reference(args):
