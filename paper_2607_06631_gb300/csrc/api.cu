@@ -1002,8 +1002,11 @@ dfs_status dfs_block_forward_host_async(dfs_plan* plan, int step, int layer, con
   // forward on the caller's stream once the inputs are in and slot b's last output is out
   DFS_CK(cudaStreamWaitEvent(st, R.loaded[b], 0));
   DFS_CK(cudaStreamWaitEvent(st, R.drained[b], 0));
-  if ((e = block_layer(plan, step, layer, R.x[b], R.t[b], R.out[b], st))) return e;
+  e = block_layer(plan, step, layer, R.x[b], R.t[b], R.out[b], st);
+  // recorded even after a failed launch, so that the slot's next input copy waits for
+  // whatever part of this forward did reach the stream (the slot is then reused next call)
   DFS_CK(cudaEventRecord(R.computed[b], st));
+  if (e) return e;
   // output: back to the host while the caller's stream moves on
   DFS_CK(cudaStreamWaitEvent(R.d2h, R.computed[b], 0));
   DFS_CK(cudaMemcpyAsync(out_host, R.out[b], bytes, cudaMemcpyDeviceToHost, R.d2h));

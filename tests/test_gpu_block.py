@@ -286,6 +286,34 @@ def test_injected_launch_failure_is_reported_and_the_plan_recovers(monkeypatch):
     np.testing.assert_array_equal(host.to_bits(out), host.to_bits(ref))
 
 
+def test_injected_launch_failure_in_the_asynchronous_host_path(monkeypatch):
+    """A launch failure inside dfs_block_forward_host_async is reported (DFS_ECUDA) and the
+    staging slot it used serves the following calls correctly."""
+    import torch
+    from paper_2607_06631_gb300 import dfs, host
+    cfg = synth.tiny()
+    shared, layers, m, acts = synth.make_problem(cfg)
+    prob = host.DeviceProblem(cfg, shared, layers, m, acts)
+    ref_plan = prob.create_plan()
+    ref = torch.empty_like(prob.x)
+    dfs.dfs_block_forward(ref_plan, 1, prob.x, prob.t_emb[1], ref)
+    dfs.dfs_plan_sync(ref_plan)
+    monkeypatch.setenv("DFS_FAULT_LAUNCH", "4")
+    plan = prob.create_plan()
+    monkeypatch.delenv("DFS_FAULT_LAUNCH")
+    x_h = prob.x.cpu().pin_memory()
+    t_h = prob.t_emb[1].cpu().pin_memory()
+    outs = [torch.zeros_like(x_h).pin_memory() for _ in range(3)]
+    with pytest.raises(dfs.DfsError) as e:
+        dfs.dfs_block_forward_host_async(plan, 1, 0, x_h, t_h, outs[0])
+    assert e.value.status == dfs.DFS_ECUDA and "injected" in str(e.value)
+    for o in outs[1:]:
+        dfs.dfs_block_forward_host_async(plan, 1, 0, x_h, t_h, o)
+    dfs.dfs_plan_sync(plan)
+    for o in outs[1:]:
+        np.testing.assert_array_equal(host.to_bits(o), host.to_bits(ref))
+
+
 def test_bounded_wait_reports_timeout_and_context_survives():
     """A wait that nothing completes gives up after about a second, the host reads
     DFS_ETIMEOUT, and the next forward on the same context is correct."""
