@@ -8,6 +8,8 @@
  *   - Linear weights are [out, in] (so every projection is y = x W^T + b).
  *   - "device" pointers are CUDA global-memory addresses of the current device; "host"
  *     pointers are ordinary CPU memory.  Nothing here takes or returns torch types.
+ *   - Every device pointer passed in must be 16-byte aligned (cudaMalloc and torch
+ *     allocations are); a misaligned one is rejected with DFS_EINVAL before any GPU work.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).  All GPU
  *     work is enqueued on it; no entry point synchronises except dfs_plan_create,
  *     dfs_plan_sync and dfs_block_forward_host, which say so.

@@ -293,6 +293,10 @@ struct ProfScope {
 
 // ------------------------------------------------------------------ validation (host only)
 
+// Device buffers are read and written with 16-byte vectors and TMA (cudaMalloc and torch
+// allocations are at least 256-byte aligned).
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
 dfs_status validate(const dfs_config* c, const dfs_layer_weights* layers, const void* w_t, const void* b_t,
                     const dfs_masks* m, const void* ctx, dfs_plan** out) {
   if (!out) return fail(DFS_EINVAL, "out is NULL");
@@ -323,14 +327,20 @@ dfs_status validate(const dfs_config* c, const dfs_layer_weights* layers, const 
     const dfs_layer_weights& w = layers[l];
     const void* req[] = {w.wq, w.bq, w.wk, w.bk, w.wv, w.bv, w.wo, w.bo, w.gq, w.gk, w.w_up, w.b_up, w.w_down,
                          w.b_down, w.e_mod};
-    for (const void* p : req)
+    for (const void* p : req) {
       if (!p) return fail(DFS_EINVAL, "layer %d: NULL weight pointer", l);
+      if (!aligned16(p)) return fail(DFS_EINVAL, "layer %d: weight pointers must be 16-byte aligned", l);
+    }
     if (c->has_cross) {
       const void* rc[] = {w.cwq, w.cbq, w.cwk, w.cbk, w.cwv, w.cbv, w.cwo, w.cbo, w.cgq, w.cgk, w.cln_w, w.cln_b};
-      for (const void* p : rc)
+      for (const void* p : rc) {
         if (!p) return fail(DFS_EINVAL, "layer %d: NULL cross-attention weight pointer", l);
+        if (!aligned16(p)) return fail(DFS_EINVAL, "layer %d: weight pointers must be 16-byte aligned", l);
+      }
     }
   }
+  if (!aligned16(w_t) || !aligned16(b_t) || (c->has_cross && !aligned16(ctx)))
+    return fail(DFS_EINVAL, "w_t, b_t and ctx must be 16-byte aligned");
   if (!m->block_gate || !m->head_gate || !m->ffn_gate) return fail(DFS_EINVAL, "NULL gate array");
   const long long TL = static_cast<long long>(c->n_steps) * c->n_layers;
   auto check01 = [](const uint8_t* g, long long n) {
@@ -884,10 +894,13 @@ dfs_status forward_impl(dfs_plan* P, int s, int l, const bf16* x, bf16* out, cud
   return DFS_OK;
 }
 
-dfs_status check_forward_args(dfs_plan* P, int step, int layer, const void* x, const void* t_emb, void* out) {
+dfs_status check_forward_args(dfs_plan* P, int step, int layer, const void* x, const void* t_emb, void* out,
+                              bool device = true) {
   if (!P) return fail(DFS_EINVAL, "plan is NULL");
   if (!x || !t_emb || !out) return fail(DFS_EINVAL, "NULL x, t_emb or out");
   if (x == out) return fail(DFS_EINVAL, "x and out must not alias");
+  if (device && (!aligned16(x) || !aligned16(t_emb) || !aligned16(out)))
+    return fail(DFS_EINVAL, "x, t_emb and out must be 16-byte aligned");
   if (step < 0 || step >= P->T) return fail(DFS_EINVAL, "step %d out of range [0, %d)", step, P->T);
   if (layer < 0 || layer >= P->L) return fail(DFS_EINVAL, "layer %d out of range [0, %d)", layer, P->L);
   return DFS_OK;
@@ -987,7 +1000,7 @@ dfs_status ring_init(dfs_plan* P) {
 
 dfs_status dfs_block_forward_host_async(dfs_plan* plan, int step, int layer, const void* x_host,
                                         const void* t_emb_host, void* out_host, void* stream) {
-  dfs_status e = check_forward_args(plan, step, layer, x_host, t_emb_host, out_host);
+  dfs_status e = check_forward_args(plan, step, layer, x_host, t_emb_host, out_host, false);
   if (e) return e;
   if ((e = ring_init(plan))) return e;
   dfs_plan::HostRing& R = plan->ring;
@@ -1017,7 +1030,7 @@ dfs_status dfs_block_forward_host_async(dfs_plan* plan, int step, int layer, con
 
 dfs_status dfs_block_forward_host(dfs_plan* plan, int step, int layer, const void* x_host, const void* t_emb_host,
                                   void* out_host, void* stream) {
-  dfs_status e = check_forward_args(plan, step, layer, x_host, t_emb_host, out_host);
+  dfs_status e = check_forward_args(plan, step, layer, x_host, t_emb_host, out_host, false);
   if (e) return e;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   // slot 0 of the asynchronous ring may still be in use by earlier asynchronous calls
@@ -1034,6 +1047,7 @@ dfs_status dfs_block_forward_host(dfs_plan* plan, int step, int layer, const voi
 
 dfs_status dfs_denoise(dfs_plan* P, void* latents, int n_steps, const void* t_embs, void* stream) {
   if (!P || !latents || !t_embs) return fail(DFS_EINVAL, "NULL plan, latents or t_embs");
+  if (!aligned16(latents) || !aligned16(t_embs)) return fail(DFS_EINVAL, "latents and t_embs must be 16-byte aligned");
   if (n_steps < 1 || n_steps > P->T) return fail(DFS_EINVAL, "n_steps must be in 1..%d", P->T);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const int d = P->cfg.dim;
@@ -1103,8 +1117,10 @@ extern "C" {
 dfs_status dfs_model_attach(dfs_plan* P, const dfs_model_weights* w, void* stream) {
   if (!P || !w) return fail(DFS_EINVAL, "NULL plan or weights");
   const void* req[] = {w->patch_w, w->patch_b, w->t_w1, w->t_b1, w->t_w2, w->t_b2, w->head_mod, w->head_w, w->head_b};
-  for (const void* q : req)
+  for (const void* q : req) {
     if (!q) return fail(DFS_EINVAL, "NULL model weight pointer");
+    if (!aligned16(q)) return fail(DFS_EINVAL, "model weight pointers must be 16-byte aligned");
+  }
   if (w->in_channels < 2 || w->in_channels % 2 != 0 || w->in_channels > 1024)
     return fail(DFS_EINVAL, "in_channels must be even, 2..1024");
   if (w->freq_dim < 8 || w->freq_dim % 8 != 0 || w->freq_dim > 8192)
@@ -1146,6 +1162,7 @@ dfs_status dfs_model_attach(dfs_plan* P, const dfs_model_weights* w, void* strea
 
 dfs_status dfs_model_forward(dfs_plan* P, int step, const void* latent, float t, void* v_out, void* stream) {
   if (!P || !latent || !v_out) return fail(DFS_EINVAL, "NULL plan, latent or v_out");
+  if (!aligned16(latent) || !aligned16(v_out)) return fail(DFS_EINVAL, "latent and v_out must be 16-byte aligned");
   if (!P->has_model) return fail(DFS_EINVAL, "no model attached (dfs_model_attach)");
   if (latent == v_out) return fail(DFS_EINVAL, "latent and v_out must not alias");
   if (step < 0 || step >= P->T) return fail(DFS_EINVAL, "step %d out of range [0, %d)", step, P->T);
@@ -1160,6 +1177,7 @@ dfs_status dfs_model_forward(dfs_plan* P, int step, const void* latent, float t,
 
 dfs_status dfs_model_denoise(dfs_plan* P, void* latent, int n_steps, const float* timesteps, void* stream) {
   if (!P || !latent || !timesteps) return fail(DFS_EINVAL, "NULL plan, latent or timesteps");
+  if (!aligned16(latent)) return fail(DFS_EINVAL, "latent must be 16-byte aligned");
   if (!P->has_model) return fail(DFS_EINVAL, "no model attached (dfs_model_attach)");
   if (n_steps < 1 || n_steps > P->T) return fail(DFS_EINVAL, "n_steps must be in 1..%d", P->T);
   cudaStream_t st = static_cast<cudaStream_t>(stream);

@@ -79,6 +79,21 @@ def test_plan_create_rejects_bad_masks_and_pointers(dfs):
     assert e.value.status == dfs.DFS_EINVAL
 
 
+def test_plan_create_rejects_misaligned_device_pointers(dfs):
+    """Device buffers are read with 16-byte vectors and TMA: an address that is not
+    16-byte aligned is refused before any CUDA call."""
+    cfg = synth.tiny()
+    layers, masks = _valid_args(dfs, cfg)
+    bad = [dict(layers[0])]
+    bad[0]["w_down"] = 24
+    with pytest.raises(dfs.DfsError) as e:
+        dfs.dfs_plan_create(cfg, bad, 16, 16, masks, None, 0)
+    assert e.value.status == dfs.DFS_EINVAL and "16-byte aligned" in dfs.dfs_last_error()
+    with pytest.raises(dfs.DfsError) as e:
+        dfs.dfs_plan_create(cfg, layers, 40, 16, masks, None, 0)
+    assert e.value.status == dfs.DFS_EINVAL and "16-byte aligned" in dfs.dfs_last_error()
+
+
 def test_forward_rejects_null_plan(dfs):
     with pytest.raises(dfs.DfsError) as e:
         dfs.dfs_block_forward(0, 0, 16, 16, 32, 0)

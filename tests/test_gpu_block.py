@@ -246,6 +246,31 @@ def test_invalid_arguments_are_rejected():
     assert e.value.status == dfs.DFS_EINVAL
 
 
+def test_misaligned_device_pointers_are_rejected_before_any_launch():
+    """x / out / t_emb / latents 8 bytes off a 16-byte boundary: DFS_EINVAL, nothing
+    launched, and the plan keeps working."""
+    import torch
+    from paper_2607_06631_gb300 import dfs, host
+    cfg = synth.tiny()
+    shared, layers, m, acts = synth.make_problem(cfg)
+    prob = host.DeviceProblem(cfg, shared, layers, m, acts)
+    plan = prob.create_plan()
+    buf = torch.zeros(prob.x.numel() + 64, dtype=prob.x.dtype, device=prob.x.device)
+    out = torch.empty_like(prob.x)
+    x8, out8 = buf.data_ptr() + 8, out.data_ptr() + 8
+    for args in ((x8, prob.t_emb[0], out), (prob.x, prob.t_emb[0], out8),
+                 (prob.x, prob.t_emb[0].data_ptr() + 8, out)):
+        with pytest.raises(dfs.DfsError) as e:
+            dfs.dfs_block_forward(plan, 0, *args)
+        assert e.value.status == dfs.DFS_EINVAL and "16-byte aligned" in str(e.value)
+    with pytest.raises(dfs.DfsError) as e:
+        dfs.dfs_denoise(plan, x8, cfg.n_steps, prob.t_emb)
+    assert e.value.status == dfs.DFS_EINVAL
+    dfs.dfs_plan_sync(plan)
+    dfs.dfs_block_forward(plan, 0, prob.x, prob.t_emb[0], out)
+    dfs.dfs_plan_sync(plan)
+
+
 def test_injected_allocation_failure(monkeypatch):
     from paper_2607_06631_gb300 import dfs, host
     cfg = synth.tiny()
