@@ -14,7 +14,10 @@
 //               issuing into one of two accumulators (2 x 256 fp32 columns per CTA), so the
 //               epilogue of tile i overlaps the main loop of tile i+1.
 //   warps 2..5  epilogue of this CTA's 128 rows: tcgen05.ld 32 columns at a time, fused bias /
-//               GELU / gated residual, predicated stores for the ragged M and N edges.
+//               GELU / gated residual, predicated stores for the ragged M and N edges.  A
+//               thread owns one output row, so every global access of a warp touches 32 rows;
+//               where bases and row pitches allow, the accesses are 256-bit (one full 32-byte
+//               sector per row per instruction) to halve the number of L1 / L2 transactions.
 // Ragged K (f_s is a multiple of 8, not of 64) is covered by TMA zero fill.
 #include "kernels.cuh"
 
@@ -40,8 +43,20 @@ __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, 
   nt = local / gsz;
 }
 
-__device__ __forceinline__ void store_bf16_row(bf16* dst, const float (&v)[32], int valid) {
-  if (valid >= 32) {
+__device__ __forceinline__ void st_global_32B(void* dst, const uint4& a, const uint4& b);
+
+// `wide`: dst is 32-byte aligned (one 256-bit store per 16 values instead of two 128-bit ones)
+__device__ __forceinline__ void store_bf16_row(bf16* dst, const float (&v)[32], int valid, bool wide = false) {
+  if (valid >= 32 && wide) {
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const uint4 a = make_uint4(pack_bf16x2(v[16 * q], v[16 * q + 1]), pack_bf16x2(v[16 * q + 2], v[16 * q + 3]),
+                                 pack_bf16x2(v[16 * q + 4], v[16 * q + 5]), pack_bf16x2(v[16 * q + 6], v[16 * q + 7]));
+      const uint4 b = make_uint4(pack_bf16x2(v[16 * q + 8], v[16 * q + 9]), pack_bf16x2(v[16 * q + 10], v[16 * q + 11]),
+                                 pack_bf16x2(v[16 * q + 12], v[16 * q + 13]), pack_bf16x2(v[16 * q + 14], v[16 * q + 15]));
+      st_global_32B(dst + 16 * q, a, b);
+    }
+  } else if (valid >= 32) {
     uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -59,7 +74,7 @@ __device__ __forceinline__ void store_bf16_row(bf16* dst, const float (&v)[32], 
   }
 }
 
-__device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int row, int col0, float (&v)[32]) {
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int row, int col0, float (&v)[32], bool wide) {
   const int valid = min(32, p.N - col0);
   if (p.bias != nullptr) {
     if (valid >= 32) {
@@ -81,7 +96,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int row, int c
 
   if (p.mode == kEpiBias) {
     if (col0 < p.split) {
-      store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, valid);
+      store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, valid, wide);
     } else {
       bf16* t = p.out_t + static_cast<long long>(col0 - p.split) * p.ldt + row;
 #pragma unroll
@@ -91,7 +106,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int row, int c
   } else if (p.mode == kEpiBiasGelu) {
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = gelu_tanh(v[j]);
-    store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, valid);
+    store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, valid, wide);
   } else {  // kEpiGatedRes
     float g[32], r[32];
     if (p.gate != nullptr) {
@@ -156,25 +171,38 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int row, int c
   }
 }
 
+// 32 bytes at a 32-byte aligned global address as two 16-byte words (one 256-bit access).
+__device__ __forceinline__ void ld_global_32B(const void* src, uint4& a, uint4& b) {
+  asm volatile("ld.global.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w), "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
+               : "l"(src));
+}
+
+__device__ __forceinline__ void st_global_32B(void* dst, const uint4& a, const uint4& b) {
+  asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(dst), "r"(a.x), "r"(a.y), "r"(a.z),
+               "r"(a.w), "r"(b.x), "r"(b.y), "r"(b.z), "r"(b.w)
+               : "memory");
+}
+
 // Raw 16-byte words of one 32-column chunk of this thread's residual row (fp32: 8 words,
-// bf16: the first 4).
+// bf16: the first 4), read with 256-bit accesses.
 __device__ __forceinline__ void load_res_chunk(int res_f32, const char* rrow, int c, uint4 (&w)[8]) {
   if (res_f32) {
-    const uint4* src = reinterpret_cast<const uint4*>(rrow + c * 128);
 #pragma unroll
-    for (int q = 0; q < 8; ++q) w[q] = src[q];
+    for (int q = 0; q < 4; ++q) ld_global_32B(rrow + c * 128 + 32 * q, w[2 * q], w[2 * q + 1]);
   } else {
-    const uint4* src = reinterpret_cast<const uint4*>(rrow + c * 64);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) w[q] = src[q];
+    for (int q = 0; q < 2; ++q) ld_global_32B(rrow + c * 64 + 32 * q, w[2 * q], w[2 * q + 1]);
   }
 }
 
-// kEpiGatedRes over one full row of a 256-column tile (row < M, all columns < N): the same
-// arithmetic as epilogue_chunk, with the residual loads of chunk c + 2 issued before chunk c
-// is processed, so that each warp keeps three chunks of loads in flight instead of waiting
-// out one memory latency per 32 columns.  The residual may be the output itself (in-place
-// update): every element is still read by its own thread before that thread writes it.
+// kEpiGatedRes over one full row of a 256-column tile (row < M, all columns < N; output and
+// residual 32-byte aligned with 32-byte multiple pitches): the same arithmetic as
+// epilogue_chunk, with 256-bit loads and stores and the residual loads of chunk c + 2
+// issued before chunk c is processed, so that each warp keeps three chunks of loads in
+// flight instead of waiting out one memory latency per 32 columns.  The residual may be the
+// output itself (in-place update): every element is still read by its own thread before
+// that thread writes it.
 __device__ __forceinline__ void epilogue_gated_row(const GemmArgs& p, int row, int colb, uint32_t taddr) {
   const char* rrow = static_cast<const char*>(p.res) +
                      (static_cast<long long>(row) * p.ldr + colb) * (p.res_f32 ? 4 : 2);
@@ -231,10 +259,24 @@ __device__ __forceinline__ void epilogue_gated_row(const GemmArgs& p, int row, i
     if (p.out_f32) {
       float* op = static_cast<float*>(p.out) + static_cast<long long>(row) * p.ldo + col0;
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
-        *reinterpret_cast<float4*>(op + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+      for (int q = 0; q < 4; ++q) {
+        const uint4 a = make_uint4(__float_as_uint(v[8 * q]), __float_as_uint(v[8 * q + 1]),
+                                   __float_as_uint(v[8 * q + 2]), __float_as_uint(v[8 * q + 3]));
+        const uint4 b = make_uint4(__float_as_uint(v[8 * q + 4]), __float_as_uint(v[8 * q + 5]),
+                                   __float_as_uint(v[8 * q + 6]), __float_as_uint(v[8 * q + 7]));
+        st_global_32B(op + 8 * q, a, b);
+      }
     } else {
-      store_bf16_row(static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0, v, 32);
+      bf16* op = static_cast<bf16*>(p.out) + static_cast<long long>(row) * p.ldo + col0;
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const uint4 a = make_uint4(pack_bf16x2(v[16 * q], v[16 * q + 1]), pack_bf16x2(v[16 * q + 2], v[16 * q + 3]),
+                                   pack_bf16x2(v[16 * q + 4], v[16 * q + 5]), pack_bf16x2(v[16 * q + 6], v[16 * q + 7]));
+        const uint4 b = make_uint4(pack_bf16x2(v[16 * q + 8], v[16 * q + 9]), pack_bf16x2(v[16 * q + 10], v[16 * q + 11]),
+                                   pack_bf16x2(v[16 * q + 12], v[16 * q + 13]),
+                                   pack_bf16x2(v[16 * q + 14], v[16 * q + 15]));
+        st_global_32B(op + 16 * q, a, b);
+      }
     }
   }
 }
@@ -359,6 +401,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   } else {
     const int sub = warp & 3;  // TMEM lane quarter this warp may access
     const int r_in_tile = static_cast<int>(rank) * kGemmBM + sub * 32 + lane;
+    // the wide epilogue reads and writes 32-byte pieces: bases and row pitches must keep them aligned
+    const int osz = p.out_f32 ? 4 : 2, rsz = p.res_f32 ? 4 : 2;
+    const bool wide_ok = ((reinterpret_cast<uintptr_t>(p.out) | reinterpret_cast<uintptr_t>(p.res)) & 31u) == 0 &&
+                         (p.ldo * osz) % 32 == 0 && (p.ldr * rsz) % 32 == 0;
+    const bool wide_out = (reinterpret_cast<uintptr_t>(p.out) & 31u) == 0 && (p.ldo * osz) % 32 == 0;
     const uint32_t tempty_leader0 = map_to_rank(&tempty[0], 0), tempty_leader1 = map_to_rank(&tempty[1], 0);
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -375,7 +422,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       }
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * kGemmBN;
       // warp-uniform choice: the TMEM loads on both paths are warp-collective
-      if (p.mode == kEpiGatedRes && kb > 0 && (nt + 1) * kGemmBN <= p.N && __all_sync(0xffffffffu, row < p.M)) {
+      if (p.mode == kEpiGatedRes && kb > 0 && (nt + 1) * kGemmBN <= p.N && wide_ok &&
+          __all_sync(0xffffffffu, row < p.M)) {
         epilogue_gated_row(p, row, nt * kGemmBN, tacc);
       } else {
         for (int c = 0; c < kGemmBN; c += 32) {
@@ -388,7 +436,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] = 0.f;
           }
-          epilogue_chunk(p, row, col0, v);
+          epilogue_chunk(p, row, col0, v, wide_out);
         }
       }
       if (kb > 0) {
