@@ -41,7 +41,7 @@ typedef enum {
   DFS_ENOMEM = 2,        /* device or host allocation failed                          */
   DFS_ECUDA = 3,         /* a CUDA runtime / driver call failed                       */
   DFS_ETIMEOUT = 4,      /* a kernel's bounded wait expired; its results are invalid   */
-  DFS_EUNSUPPORTED = 5   /* valid request this build does not implement                */
+  DFS_EUNSUPPORTED = 5   /* valid request the library does not implement               */
 } dfs_status;
 
 /* How a plan holds the weights of the retained units (Sec. 4.3, Fig. 1(c)).
