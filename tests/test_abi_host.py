@@ -112,3 +112,27 @@ def test_soft_mask_gate_rules_match_oracle(dfs, kind, unit):
     ref = O.gates_from_soft_masks({0: "block", 1: "head", 2: "ffn"}[kind], m, unit)
     np.testing.assert_array_equal(g, ref)
     assert g[0, 0] == 0
+
+
+def test_header_and_c_example_are_plain_c(tmp_path):
+    """include/dfs.h is a C header (no C++ or torch types): it and the plain-C example compile
+    as strict C99 with warnings as errors, and the header also as C++17."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no gcc")
+    inc = os.path.join(ROOT, "include")
+    src = tmp_path / "h.c"
+    src.write_text('#include "dfs.h"\nint main(void) { dfs_plan* p = 0; (void)p; return 0; }\n')
+    for cmd in ([gcc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic", "-fsyntax-only", "-I", inc, str(src)],
+                ["g++", "-std=c++17", "-Wall", "-Werror", "-fsyntax-only", "-I", inc, "-x", "c++", str(src)]):
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr
+    cuda_inc = next((d for d in ("/usr/local/cuda/include",) if os.path.exists(os.path.join(d, "cuda_runtime_api.h"))),
+                    None)
+    if cuda_inc:
+        ex = os.path.join(ROOT, "paper_2607_06631_gb300", "examples", "block_forward.c")
+        r = subprocess.run([gcc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I", inc, "-I", cuda_inc, ex],
+                           capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr
