@@ -979,7 +979,7 @@ dfs_status ring_join(dfs_plan* P, cudaStream_t st) {
 dfs_status ring_init(dfs_plan* P) {
   dfs_plan::HostRing& R = P->ring;
   if (R.ready) return DFS_OK;
-  const long long n = P->N * P->cfg.dim;
+  const long long n = static_cast<long long>(P->N) * P->cfg.dim;
   R.x[0] = P->stage_x;
   R.out[0] = P->stage_out;
   R.t[0] = P->stage_t;
