@@ -266,18 +266,24 @@ def load_problem_f64(cfg):
 CPU_ROWS = 32
 
 
+def cpu_rows(cfg) -> int:
+    """Query rows of one oracle sample: the whole block for small token counts, else 32."""
+    return cfg.n_tokens if cfg.n_tokens <= 4096 else CPU_ROWS
+
+
 def cpu_baseline(cfg):
     import oracle as O
     prob = load_problem_f64(cfg)
     step = cfg.n_steps - 1
-    dt, fl = oracle_sample(cfg, prob, step, CPU_ROWS)
+    rows = cpu_rows(cfg)
+    dt, fl = oracle_sample(cfg, prob, step, rows)
     # the whole block of that step at the sample's FLOP rate (an extrapolation, not a run)
     h_s, f_s = cfg.heads_kept[step][0], 8 * cfg.chunks_kept[step][0]
     hc = cfg.xheads_kept[step][0] if cfg.has_cross else 0
     full = O.block_flops(cfg.n_tokens, cfg.dim, cfg.head_dim, h_s, f_s, hc, cfg.ctx_len)
     return {"value": fl / dt / 1e12, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
             "sample": "float64 oracle, MoM step %d, %d query rows (keys/values over all %d tokens): "
-                      "%.3e counted FLOPs in %.1f s" % (step, CPU_ROWS, cfg.n_tokens, fl, dt),
+                      "%.3e counted FLOPs in %.1f s" % (step, rows, cfg.n_tokens, fl, dt),
             "block_seconds_extrapolated": round(full / (fl / dt), 2),
             "extrapolation": "one full block of MoM step %d (%.3e algorithmic FLOPs) at the sample's FLOP rate"
                              % (step, full)}
@@ -289,11 +295,12 @@ def run_reference(args):
         return 0
     cfg = get_config(args.config, args.grid)
     prob = load_problem_f64(cfg)
+    rows = cpu_rows(cfg)
     for i in range(args.warmup):
-        oracle_sample(cfg, prob, i % cfg.n_steps, CPU_ROWS, seed=1000 + i)
+        oracle_sample(cfg, prob, i % cfg.n_steps, rows, seed=1000 + i)
     tot_t = tot_f = 0.0
     for i in range(args.steps):
-        dt, fl = oracle_sample(cfg, prob, i % cfg.n_steps, CPU_ROWS, seed=i)
+        dt, fl = oracle_sample(cfg, prob, i % cfg.n_steps, rows, seed=i)
         tot_t += dt
         tot_f += fl
     val = tot_f / tot_t / 1e12
@@ -303,7 +310,7 @@ def run_reference(args):
             "data": "synthetic", "config": {"workload": workload_desc(cfg)},
             "cpu_baseline": {"kind": "oracle", "cores": cpu_cores(), "value": val, "unit": "TFLOP/s",
                              "sample": "each step: float64 oracle on one MoM step (cycling 0..3), %d query "
-                                       "rows, keys/values over all %d tokens" % (CPU_ROWS, cfg.n_tokens)},
+                                       "rows, keys/values over all %d tokens" % (rows, cfg.n_tokens)},
             "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
