@@ -219,7 +219,7 @@ struct QkParams {
 // memory from the per-band tables while the row loads, and the q and k statistics share one
 // reduction.
 template <int VPT>
-__global__ void __launch_bounds__(kQkThreads, 4) qk_norm_rope_kernel(const QkParams p) {
+__global__ void __launch_bounds__(kQkThreads, 6) qk_norm_rope_kernel(const QkParams p) {
   __shared__ float red[2][32];
   __shared__ float rcos[64], rsin[64];
   const long long row = blockIdx.x;
