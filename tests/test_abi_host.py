@@ -100,6 +100,28 @@ def test_forward_rejects_null_plan(dfs):
     assert e.value.status == dfs.DFS_EINVAL
 
 
+@pytest.mark.parametrize("call", ["layer", "host", "host_async", "noalloc", "denoise", "model_forward",
+                                  "model_denoise", "sync", "memory", "flops"])
+def test_every_entry_point_rejects_a_null_plan_before_any_cuda_call(dfs, call):
+    import numpy as np
+    h = np.zeros(64, dtype=np.uint16)
+    calls = {
+        "layer": lambda: dfs.dfs_block_forward_layer(0, 0, 0, 16, 16, 32, 0),
+        "host": lambda: dfs.dfs_block_forward_host(0, 0, 0, h, h[:16], h[32:], 0),
+        "host_async": lambda: dfs.dfs_block_forward_host_async(0, 0, 0, h, h[:16], h[32:], 0),
+        "noalloc": lambda: dfs.dfs_block_forward_noalloc(0, 0, 0, 16, 16, 32, 0),
+        "denoise": lambda: dfs.dfs_denoise(0, 16, 4, 32, 0),
+        "model_forward": lambda: dfs.dfs_model_forward(0, 0, 16, 1.0, 32, 0),
+        "model_denoise": lambda: dfs.dfs_model_denoise(0, 16, 4, [1000.0, 750.0, 500.0, 250.0], 0),
+        "sync": lambda: dfs.dfs_plan_sync(0, 0),
+        "memory": lambda: dfs.dfs_plan_memory(0),
+        "flops": lambda: dfs.dfs_plan_flops(0, 0, 0),
+    }
+    with pytest.raises(dfs.DfsError) as e:
+        calls[call]()
+    assert e.value.status == dfs.DFS_EINVAL
+
+
 @pytest.mark.parametrize("kind,unit", [(0, 1), (1, 64), (1, 128), (2, 1)])
 def test_soft_mask_gate_rules_match_oracle(dfs, kind, unit):
     rng = np.random.default_rng(kind * 100 + unit)
