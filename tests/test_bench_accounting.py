@@ -54,3 +54,20 @@ def test_hbm_units_are_the_stated_byte_counts():
     hsum = sum(cfg.heads_kept[s][0] for s in range(cfg.n_steps)) * cfg.head_dim
     assert units["qk_norm_rope"] == 2.0 * N * 2 * hsum * 2
     assert units["modulation"] == cfg.n_steps * 6.0 * d * d * 2
+
+
+def test_reference_arm_prints_one_contract_line_on_the_tiny_block():
+    """`bench.py --impl reference` (the oracle timed on the host cores) prints one JSON line with
+    the contract's keys; on the tiny configuration each step is the whole block."""
+    import json
+    import subprocess
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "tiny",
+                        "--steps", "1", "--warmup", "0"], capture_output=True, text=True, timeout=600, cwd=ROOT)
+    assert r.returncode == 0, r.stderr
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["unit"] == "TFLOP/s" and d["value"] > 0 and d["higher_is_better"]
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
+    assert "512 query rows" in d["cpu_baseline"]["sample"]
