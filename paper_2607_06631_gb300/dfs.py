@@ -120,6 +120,7 @@ def lib() -> ctypes.CDLL:
 
 
 def dfs_last_error() -> str:
+    """Message of the calling thread's last failed call (empty if none)."""
     return lib().dfs_last_error().decode()
 
 
@@ -224,15 +225,18 @@ def dfs_plan_create(cfg, layers: Sequence[Dict[str, Any]], w_t, b_t, masks: Dict
 
 
 def dfs_block_forward(plan, step: int, x, t_emb, out, stream=None):
+    """Layer 0 of the plan at MoM step `step`: out = block(x, t_emb) (bf16 device buffers [N, dim], [dim])."""
     _check(lib().dfs_block_forward(_h(plan), step, _ptr(x), _ptr(t_emb), _ptr(out), _stream(stream)))
 
 
 def dfs_block_forward_layer(plan, step: int, layer: int, x, t_emb, out, stream=None):
+    """As dfs_block_forward for layer `layer` of the plan."""
     _check(lib().dfs_block_forward_layer(_h(plan), step, layer, _ptr(x), _ptr(t_emb), _ptr(out),
                                          _stream(stream)))
 
 
 def dfs_block_forward_host(plan, step: int, layer: int, x_host, t_emb_host, out_host, stream=None):
+    """As dfs_block_forward_layer on HOST buffers (pinned for full copy speed); synchronises `stream`."""
     _check(lib().dfs_block_forward_host(_h(plan), step, layer, _ptr(x_host), _ptr(t_emb_host),
                                         _ptr(out_host), _stream(stream)))
 
@@ -251,6 +255,7 @@ def dfs_block_forward_noalloc(plan, step: int, layer: int, x, t_emb, out, stream
 
 
 def dfs_denoise(plan, latents, n_steps: int, t_embs, stream=None):
+    """Few-step loop on device latents [N, dim] in place: every layer of each step, then x += out / T."""
     _check(lib().dfs_denoise(_h(plan), _ptr(latents), n_steps, _ptr(t_embs), _stream(stream)))
 
 
@@ -264,10 +269,12 @@ def dfs_model_attach(plan, weights: Dict[str, Any], in_channels: int = 16, freq_
 
 
 def dfs_model_forward(plan, step: int, latent, t: float, v_out, stream=None):
+    """One pass of the attached Wan-shaped model at step `step` and timestep t: latent -> velocity v_out."""
     _check(lib().dfs_model_forward(_h(plan), step, _ptr(latent), float(t), _ptr(v_out), _stream(stream)))
 
 
 def dfs_model_denoise(plan, latent, n_steps: int, timesteps: Sequence[float], stream=None):
+    """Few-step latent denoise with the attached model; `timesteps` holds one host float per step."""
     ts = np.ascontiguousarray(timesteps, dtype=np.float32)
     _check(lib().dfs_model_denoise(_h(plan), _ptr(latent), n_steps, ts.ctypes.data, _stream(stream)))
 
@@ -309,12 +316,14 @@ def dfs_plan_memory(plan):
 
 
 def dfs_plan_flops(plan, step: int, layer: int = 0) -> float:
+    """Algorithmic FLOPs of (step, layer) (closed form, 2 per multiply-add)."""
     f = ctypes.c_double()
     _check(lib().dfs_plan_flops(_h(plan), step, layer, ctypes.byref(f)))
     return f.value
 
 
 def dfs_plan_workspace(plan, which):
+    """Device address, shape and dtype of a workspace buffer of the last forward (test hook)."""
     w = WORKSPACE[which] if isinstance(which, str) else which
     p, r, c, ld, dt = ctypes.c_void_p(), ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int()
     _check(lib().dfs_plan_workspace(_h(plan), w, ctypes.byref(p), ctypes.byref(r), ctypes.byref(c),
@@ -323,14 +332,17 @@ def dfs_plan_workspace(plan, which):
 
 
 def dfs_plan_sync(plan, stream=None):
+    """Waits for `stream` (and the asynchronous host path's copies); raises on a kernel's bounded-wait timeout."""
     _check(lib().dfs_plan_sync(_h(plan), _stream(stream)))
 
 
 def dfs_selftest_wait_timeout(plan, stream=None):
+    """Launches a kernel whose bounded wait runs out on purpose (the timeout path's test hook)."""
     _check(lib().dfs_selftest_wait_timeout(_h(plan), _stream(stream)))
 
 
 def dfs_plan_profile(plan, enable: bool):
+    """Turns per-kernel CUDA-event timing of the plan's launches on or off."""
     _check(lib().dfs_plan_profile(_h(plan), 1 if enable else 0))
 
 
@@ -353,6 +365,7 @@ def dfs_gates_from_soft_masks(kind: int, m: np.ndarray, unit_size: int = 1) -> n
 
 
 def dfs_plan_destroy(plan):
+    """Frees the plan and everything it owns."""
     if isinstance(plan, Plan):
         plan.close()
     elif plan:
