@@ -57,6 +57,7 @@ __all__ = [
     "linear", "modulation", "layer_norm", "adaln", "rms_norm", "rope_pairs", "rope_angles",
     "apply_rope", "attention", "gelu_tanh", "block_forward_masked",
     "block_forward_compacted", "block_flops", "denoise", "MacCounter",
+    "cross_input_norm", "output_head",
     "patchify", "unpatchify", "timestep_embedding", "time_mlp", "model_forward", "model_denoise",
 ]
 
@@ -379,7 +380,8 @@ def block_forward_masked(cfg, shared, lw, masks, step: int, layer: int, x, t_emb
     x1 = x1 + g_a * linear(o, lw["wo"], lw["bo"])
 
     if cfg.has_cross:
-        x1 = x1 + _cross_masked(cfg, lw, masks, step, layer, x1, ctx)
+        inter["x1a"] = x1
+        x1 = x1 + _cross_masked(cfg, lw, masks, step, layer, x1, ctx, inter)
 
     xm2 = adaln(x1, sh_f, sc_f, eps)
     u = gelu_tanh(linear(xm2, lw["w_up"], lw["b_up"]))
@@ -391,14 +393,22 @@ def block_forward_masked(cfg, shared, lw, masks, step: int, layer: int, x, t_emb
     return out
 
 
-def _cross_masked(cfg, lw, masks, step, layer, x1, ctx):
+def cross_input_norm(x1, cln_w, cln_b, eps: float) -> np.ndarray:
+    """Input of the cross-attention (R6): an affine LayerNorm of the residual x1,
+    LN(x1) * cln_w + cln_b, with the LayerNorm of R3."""
+    return layer_norm(x1, eps, cln_w, cln_b)
+
+
+def _cross_masked(cfg, lw, masks, step, layer, x1, ctx, inter=None):
     d, H, dh, eps = cfg.dim, cfg.n_heads, cfg.head_dim, cfg.ln_eps
     xg = masks.get("xhead_gate")
     hg = np.ones(H) if xg is None else xg[step, layer].astype(np.float64)
     if hg.sum() == 0:
         return np.zeros_like(x1) + lw["cbo"]
     keep = np.repeat(hg, dh)
-    xc = layer_norm(x1, eps, lw["cln_w"], lw["cln_b"])
+    xc = cross_input_norm(x1, lw["cln_w"], lw["cln_b"], eps)
+    if inter is not None:
+        inter["xc"] = xc
     q = rms_norm(linear(xc, lw["cwq"], lw["cbq"]), lw["cgq"], keep, eps, cfg.qk_norm_mode, dh)
     k = rms_norm(linear(ctx, lw["cwk"], lw["cbk"]), lw["cgk"], keep, eps, cfg.qk_norm_mode, dh)
     v = linear(ctx, lw["cwv"], lw["cbv"])
@@ -445,7 +455,8 @@ def block_forward_compacted(cfg, shared, lw, masks, step: int, layer: int, x, t_
         x1 = xr + g_a * lw["bo"]
 
     if cfg.has_cross:
-        x1 = x1 + _cross_compacted(cfg, lw, P, idx, x1, ctx, counter)
+        inter["x1a"] = x1
+        x1 = x1 + _cross_compacted(cfg, lw, P, idx, x1, ctx, counter, inter)
         inter["x1c"] = x1
 
     xm2 = adaln(x1, sh_f, sc_f, eps)
@@ -461,14 +472,16 @@ def block_forward_compacted(cfg, shared, lw, masks, step: int, layer: int, x, t_
     return out
 
 
-def _cross_compacted(cfg, lw, P, idx, x1, ctx, counter):
+def _cross_compacted(cfg, lw, P, idx, x1, ctx, counter, inter=None):
     dh, eps = cfg.head_dim, cfg.ln_eps
     hc = len(idx["xheads"])
     if hc == 0:
         return np.zeros_like(x1) + lw["cbo"]
     hd = hc * dh
     ones = np.ones(hd)
-    xc = layer_norm(x1, eps, lw["cln_w"], lw["cln_b"])
+    xc = cross_input_norm(x1, lw["cln_w"], lw["cln_b"], eps)
+    if inter is not None:
+        inter["xc"] = xc
     q = rms_norm(linear(xc, P["cwq"], P["cbq"], counter), P["cgq"], ones, eps, cfg.qk_norm_mode, dh)
     kv = linear(ctx, P["cwkv"], P["cbkv"], counter)
     k = rms_norm(kv[:, :hd], P["cgk"], ones, eps, cfg.qk_norm_mode, dh)
@@ -558,6 +571,15 @@ def time_mlp(mw, t: float) -> np.ndarray:
     return mw["t_w2"] @ h + mw["t_b2"]
 
 
+def output_head(x, head_mod, t_emb, head_w, head_b, eps: float) -> np.ndarray:
+    """Output head of the model (R18) on token rows x [n, d]: shift_h = head_mod[0] + t_emb,
+    scale_h = head_mod[1] + t_emb, y = LN(x) (1 + scale_h) + shift_h, returns y W_h^T + b_h
+    ([n, 4 C], still in token layout)."""
+    shift = head_mod[0] + t_emb
+    scale = head_mod[1] + t_emb
+    return linear(adaln(x, shift, scale, eps), head_w, head_b)
+
+
 def model_forward(cfg, shared, layers, mw, masks, step: int, latent, t: float, ctx=None, want: bool = False):
     """One pass of the Wan-shaped model at denoising step `step` (R16-R18): patch embedding,
     every block with its step-`step` structure (masked-dense form), output head; returns the
@@ -566,10 +588,8 @@ def model_forward(cfg, shared, layers, mw, masks, step: int, latent, t: float, c
     x = linear(patchify(latent), mw["patch_w"], mw["patch_b"])
     for l in range(cfg.n_layers):
         x = block_forward_masked(cfg, shared, layers[l], masks, step, l, x, t_emb, ctx)
-    shift = mw["head_mod"][0] + t_emb
-    scale = mw["head_mod"][1] + t_emb
-    y = adaln(x, shift, scale, cfg.ln_eps)
-    v = unpatchify(linear(y, mw["head_w"], mw["head_b"]), latent.shape)
+    v = unpatchify(output_head(x, mw["head_mod"], t_emb, mw["head_w"], mw["head_b"], cfg.ln_eps),
+                   latent.shape)
     return (v, {"t_emb": t_emb, "x_last": x}) if want else v
 
 

@@ -132,6 +132,5 @@ def test_wan13b_shaped_one_layer_model_full_size():
         t_emb = O.time_mlp(MW, ts[s])
         x = O.linear(O.patchify(lat), MW["patch_w"], MW["patch_b"])
         xo = O.block_forward_masked(cfg, W, LW[0], m, s, 0, x, t_emb, X["ctx"], rows=rows)
-        y = O.adaln(xo, MW["head_mod"][0] + t_emb, MW["head_mod"][1] + t_emb, cfg.ln_eps)
-        ref = O.linear(y, MW["head_w"], MW["head_b"])
+        ref = O.output_head(xo, MW["head_mod"], t_emb, MW["head_w"], MW["head_b"], cfg.ln_eps)
         assert rel_err(got, ref) <= TOL, (s, rel_err(got, ref))

@@ -89,6 +89,14 @@ def _gelu_coefficient(orig):
     return lambda x: 0.5 * x * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (x + 0.0447 * x ** 2)))
 
 
+def _cross_ln_weight_bias_swapped(orig):
+    return lambda x1, cln_w, cln_b, eps: orig(x1, cln_b, cln_w, eps)
+
+
+def _head_shift_scale_swapped(orig):
+    return lambda x, head_mod, t_emb, head_w, head_b, eps: orig(x, head_mod[::-1], t_emb, head_w, head_b, eps)
+
+
 MUTATIONS = {
     "LayerNorm with the unbiased variance": ("layer_norm", _ln_unbiased),
     "adaLN scale without the 1 +": ("adaln", _adaln_no_one),
@@ -102,6 +110,8 @@ MUTATIONS = {
     "linear with W not transposed": ("linear", _linear_transposed),
     "shift and scale swapped": ("modulation", _modulation_swapped),
     "timestep sinusoid halves swapped": ("timestep_embedding", _time_cos_sin_swapped),
+    "cross-attention LayerNorm weight and bias swapped": ("cross_input_norm", _cross_ln_weight_bias_swapped),
+    "output head shift and scale swapped": ("output_head", _head_shift_scale_swapped),
 }
 
 

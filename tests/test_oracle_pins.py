@@ -386,6 +386,59 @@ def test_modulation_vectors_land_where_read():
     np.testing.assert_allclose(it["xm2"], np.tile(base[3] + e[3], (cfg.n_tokens, 1)), atol=1e-12)
 
 
+def _cross_branch(fn, cfg, W, lw, M, s, X):
+    """The cross-attention branch of one block (R6): x1 after the cross-attention minus x1
+    before it, with the cross-attention's input and its LayerNorm output."""
+    _, it = fn(cfg, W, lw, M, s, 0, X["x"], X["t_emb"][s], X["ctx"], want=True)
+    return it["x1"] - it["x1a"], it["x1a"], it["xc"]
+
+
+@pytest.mark.parametrize("form", ["masked", "compacted"])
+def test_cross_layer_norm_weight_zero_gives_one_query_row(form):
+    """R6 with cln_w = 0: LN(x1) cln_w + cln_b = cln_b for every token, so every query row is
+    the same, the branch is one row repeated, and that row is the softmax of a single query
+    over the context keys (brute force) projected by Wo_c."""
+    fn = O.block_forward_masked if form == "masked" else O.block_forward_compacted
+    cfg, W, LW, M, X = _problem(has_cross=1)
+    lw = dict(LW[0])
+    lw["cln_w"] = np.zeros_like(lw["cln_w"])
+    s = 1
+    br, x1a, xc = _cross_branch(fn, cfg, W, lw, M, s, X)
+    np.testing.assert_array_equal(xc, np.tile(lw["cln_b"], (x1a.shape[0], 1)))
+    np.testing.assert_allclose(br, np.tile(br[0], (br.shape[0], 1)), rtol=0, atol=1e-12 * np.abs(br).max())
+    # the one row by hand: retained cross heads, full-row RMSNorm over their channels (R4 mode 0)
+    H, dh, eps = cfg.n_heads, cfg.head_dim, cfg.ln_eps
+    heads = np.flatnonzero(M["xhead_gate"][s, 0])
+    r = (heads[:, None] * dh + np.arange(dh)[None, :]).reshape(-1)
+
+    def rms(a, g):
+        return a / np.sqrt((a ** 2).mean(-1, keepdims=True) + eps) * g
+
+    q = rms(lw["cwq"][r] @ lw["cln_b"] + lw["cbq"][r], lw["cgq"][r])
+    k = rms(X["ctx"] @ lw["cwk"][r].T + lw["cbk"][r], lw["cgk"][r])
+    v = X["ctx"] @ lw["cwv"][r].T + lw["cbv"][r]
+    L, h = X["ctx"].shape[0], len(heads)
+    o = _attention_brute(q.reshape(1, h, dh), k.reshape(L, h, dh), v.reshape(L, h, dh)).reshape(-1)
+    want = lw["cwo"][:, r] @ o + lw["cbo"]
+    np.testing.assert_allclose(br[0], want, rtol=1e-10, atol=1e-12)
+
+
+@pytest.mark.parametrize("form", ["masked", "compacted"])
+def test_cross_layer_norm_is_the_library_affine_layer_norm(form):
+    """R6: the cross-attention reads torch's affine LayerNorm of x1 (weight cln_w, bias cln_b);
+    with cln_w = 1 and cln_b = 0 that is the plain LayerNorm."""
+    torch = pytest.importorskip("torch")
+    fn = O.block_forward_masked if form == "masked" else O.block_forward_compacted
+    cfg, W, LW, M, X = _problem(has_cross=1)
+    d = cfg.dim
+    for w, b in ((LW[0]["cln_w"], LW[0]["cln_b"]), (np.ones(d), np.zeros(d))):
+        lw = dict(LW[0], cln_w=w, cln_b=b)
+        _, x1a, xc = _cross_branch(fn, cfg, W, lw, M, 2, X)
+        ref = torch.nn.functional.layer_norm(torch.from_numpy(x1a), (d,), torch.from_numpy(w),
+                                             torch.from_numpy(b), eps=cfg.ln_eps).numpy()
+        np.testing.assert_allclose(xc, ref, rtol=1e-12, atol=1e-12)
+
+
 # --------------------------------------------------------------------------- FLOPs
 
 @pytest.mark.parametrize("has_cross", [0, 1])
@@ -498,6 +551,37 @@ def test_model_head_reads_only_its_bias_when_its_weights_vanish():
     v = O.model_forward(cfg, W, LW, mw, M, 1, lat, 750.0, X["ctx"])
     want = O.unpatchify(np.tile(mw["head_b"], (cfg.n_tokens, 1)), lat.shape)
     np.testing.assert_allclose(v, want, rtol=0, atol=0)
+
+
+def test_model_head_scale_minus_one_returns_the_shift():
+    """R18: with head_mod[1] = -1 - t_emb the head's 1 + scale_h vanishes, so every token's
+    head input is shift_h = head_mod[0] + t_emb and the velocity is that one row projected."""
+    cfg, W, LW, M, X, mw, lat = _model_problem()
+    t = 500.0
+    t_emb = O.time_mlp(mw, t)
+    mw = dict(mw)
+    hm = mw["head_mod"].copy()
+    hm[1] = -1.0 - t_emb
+    mw["head_mod"] = hm
+    v = O.model_forward(cfg, W, LW, mw, M, 2, lat, t, X["ctx"])
+    row = mw["head_w"] @ (hm[0] + t_emb) + mw["head_b"]
+    want = O.unpatchify(np.tile(row, (cfg.n_tokens, 1)), lat.shape)
+    np.testing.assert_allclose(v, want, rtol=1e-12, atol=1e-12)
+
+
+def test_model_head_without_modulation_is_the_library_layer_norm():
+    """R18: with shift_h = scale_h = 0 (head_mod = -t_emb in both rows) the head is torch's
+    plain LayerNorm of the last block's output followed by the head projection."""
+    torch = pytest.importorskip("torch")
+    cfg, W, LW, M, X, mw, lat = _model_problem()
+    t = 250.0
+    t_emb = O.time_mlp(mw, t)
+    mw = dict(mw)
+    mw["head_mod"] = np.stack([-t_emb, -t_emb])
+    v, it = O.model_forward(cfg, W, LW, mw, M, 3, lat, t, X["ctx"], want=True)
+    y = torch.nn.functional.layer_norm(torch.from_numpy(it["x_last"]), (cfg.dim,), eps=cfg.ln_eps).numpy()
+    want = O.unpatchify(y @ mw["head_w"].T + mw["head_b"], lat.shape)
+    np.testing.assert_allclose(v, want, rtol=1e-10, atol=1e-12)
 
 
 def test_model_blocks_off_leave_the_embedded_patches():
