@@ -16,11 +16,11 @@
  *   - Errors are returned as dfs_status and never thrown across the ABI; dfs_last_error()
  *     gives a message for the calling thread.  On any error nothing is written to `out`.
  *   - A plan may be used from one host thread at a time.
- *   - CUDA graphs: dfs_block_forward, dfs_block_forward_layer, dfs_block_forward_noalloc
- *     (after its first call on the device), dfs_denoise, dfs_model_forward and
- *     dfs_model_denoise enqueue only kernel launches and device-to-device copies, with no
- *     allocation and no synchronisation, so a call made while `stream` is capturing
- *     (cudaStreamBeginCapture) is recorded into the graph.  A replay reuses the pointers
+ *   - CUDA graphs: dfs_block_forward, dfs_block_forward_layer, dfs_denoise,
+ *     dfs_model_forward and dfs_model_denoise enqueue only kernel launches and
+ *     device-to-device copies, with no allocation and no synchronisation, so a call made
+ *     while `stream` is capturing (cudaStreamBeginCapture) is recorded into the graph.
+ *     A replay reuses the pointers
  *     and host scalars (timesteps) of the capture and reads the device buffers' contents at
  *     replay time.  Per-kernel profiling (dfs_plan_profile) must be off while capturing.
  */
@@ -117,6 +117,10 @@ dfs_status dfs_plan_create(const dfs_config* cfg, const dfs_layer_weights* layer
                            const void* ctx, void* stream, dfs_plan** out);
 
 /* Forward of layer 0 at denoising step `step` (0-based; the paper's t_{step+1}).
+ * Defined by Eq. 2 (Sec. 3.2: each gated head / FFN chunk / block output multiplied by
+ * its binary gate), the export of the gated network to a dense per-step model (Sec. 3.2)
+ * and the per-step index-table engine over the union super-model (Sec. 4.3, Fig. 1(c)):
+ * the pruned units are never computed, and the result equals the masked dense block.
  * x, out: [N, dim] bf16 device, caller-owned, must not alias.  t_emb: [dim] bf16
  * device.  Computes, with the step's compacted weights only:
  *   mod = W_t t_emb + b_t + E_l; xm = LN(x)(1+scale_a)+shift_a; qkv = xm Wqkv_s^T + b;
@@ -127,7 +131,8 @@ dfs_status dfs_plan_create(const dfs_config* cfg, const dfs_layer_weights* layer
 dfs_status dfs_block_forward(dfs_plan* plan, int step, const void* x, const void* t_emb,
                              void* out, void* stream);
 
-/* As dfs_block_forward for any layer of the plan. */
+/* As dfs_block_forward for any layer of the plan (same passages: Eq. 2, the Sec. 3.2
+ * export, Sec. 4.3; each layer has its own gates and index tables per step). */
 dfs_status dfs_block_forward_layer(dfs_plan* plan, int step, int layer, const void* x,
                                    const void* t_emb, void* out, void* stream);
 
@@ -157,20 +162,32 @@ dfs_status dfs_block_forward_host_async(dfs_plan* plan, int step, int layer, con
                                         const void* t_emb_host, void* out_host, void* stream);
 
 /* Allocation-free variant of dfs_block_forward_layer (the paper has no counterpart;
- * this is a deployment convenience).  Same arguments, same kernels, same result; the
- * per-call activation workspace lives in a 16 MiB device array that the library
- * declares statically, instead of memory the plan allocated.  For callers that must not
- * allocate device memory while running the model: a host application that owns every
- * device allocation through its own pool and budget, or a latency-critical loop that
- * cannot absorb cudaMalloc's implicit synchronisation.  The plan must already exist.
- *   - Nothing is allocated: no cudaMalloc, cudaFree or allocating library routine.
- *   - The first call on a device looks up the array's device address (with that device
- *     current) and keeps it; make that first call before any stream capture.
+ * this is a deployment convenience).  Same arguments, same kernels in the same order,
+ * bit-identical result; the per-call activation workspace lives in a 16 MiB device array
+ * that the library declares statically, instead of memory the plan allocated.  For
+ * callers that must not allocate device memory while running the model: a host
+ * application that owns every device allocation through its own pool and budget, or a
+ * latency-critical loop that cannot absorb cudaMalloc's implicit synchronisation.  The
+ * plan must already exist, and its device must be the current one (else DFS_EINVAL).
+ *   - Nothing is allocated: no cudaMalloc, cudaFree or allocating library routine.  The
+ *     TMA descriptors of the workspace operands are encoded on the host at every call
+ *     (a few microseconds of CPU time, no device work).
+ *   - The first call on a device after a plan was created there looks up the array's
+ *     device address (with that device current) and keeps it; make that call before
+ *     any stream capture.  dfs_plan_create drops the kept address, because a device
+ *     reset (which also invalidates every earlier plan) may move the array.
  *   - Every call on a device shares the one array and leaves its contents behind; no
  *     call relies on what an earlier call left.  Calls whose GPU work overlaps (other
  *     streams, other host threads) race on the array: serialise them.
- *   - A (step, layer) whose workspace (about N * (6 dim + 8 h_s head_dim + 2 f_s) bytes)
- *     exceeds 16 MiB is rejected with DFS_EUNSUPPORTED and a message giving the need.
+ *   - Under DFS_ENGINE_UNION the step's FFN panels are still gathered into the plan's
+ *     own FFN scratch pair (allocated by dfs_plan_create), as in every forward of that
+ *     plan: a call also races with any other forward of the same plan whose GPU work
+ *     overlaps it.
+ *   - Workspace of a (step, layer), with h = h_s head_dim, c = hc head_dim (cross heads,
+ *     0 without cross-attention), f = f_s and every term rounded up to 256 bytes:
+ *       24 dim + 2 N dim + 4 N h + 2 h ceil64(N) + 2 N max(h, c) + 4 N dim + 2 N f + 2 N c
+ *     bytes; above 16 MiB (16777216 bytes) the call is rejected with DFS_EUNSUPPORTED and
+ *     a message giving the need.
  * Errors: as dfs_block_forward_layer, plus DFS_EUNSUPPORTED. */
 dfs_status dfs_block_forward_noalloc(dfs_plan* plan, int step, int layer, const void* x,
                                      const void* t_emb, void* out, void* stream);
@@ -220,7 +237,9 @@ dfs_status dfs_model_denoise(dfs_plan* plan, void* latent, int n_steps, const fl
 
 /* Test hooks ---------------------------------------------------------------------- */
 
-/* Index lists of I_t for (step, layer).  kind: 0 = retained head ids, 1 = retained FFN
+/* Index lists of I_t for (step, layer): the per-step index table of Sec. 4.3 / Fig. 1(c),
+ * built from the hard gates of Sec. 4.1 (FFN chunks of C = 8 channels, App. A).
+ * kind: 0 = retained head ids, 1 = retained FFN
  * chunk ids, 2 = retained cross-attention head ids; 3, 4, 5 = the ids of the layer's
  * union super-model (heads / FFN chunks / cross heads retained at any step of the plan,
  * independent of `step`); 6, 7, 8 = the positions of the step's retained heads / chunks /
@@ -229,8 +248,9 @@ dfs_status dfs_model_denoise(dfs_plan* plan, void* latent, int n_steps, const fl
 dfs_status dfs_plan_indices(const dfs_plan* plan, int step, int layer, int kind,
                             int32_t* out, int* count);
 
-/* Device address and shape of a compacted panel (bf16, row-major, leading dim *ld in
- * elements).  which: 0 Wqkv [3 h_s dh, dim], 1 bqkv [3 h_s dh], 2 gq [h_s dh],
+/* Device address and shape of a compacted panel: the dense per-step weights of the
+ * exported model (Sec. 3.2), i.e. the active parameters of step t gathered through I_t
+ * (Sec. 4.3, Fig. 1(c)); bf16, row-major, leading dim *ld in elements.  which: 0 Wqkv [3 h_s dh, dim], 1 bqkv [3 h_s dh], 2 gq [h_s dh],
  * 3 gk [h_s dh], 4 Wo [dim, h_s dh], 5 W_up [f_s, dim], 6 b_up [f_s],
  * 7 W_down [dim, f_s]; cross: 8 cWq [hc dh, dim], 9 cbq, 10 cWkv [2 hc dh, dim],
  * 11 cbkv, 12 cgq, 13 cgk, 14 cWo [dim, hc dh].  A panel with zero rows or columns
@@ -254,7 +274,12 @@ dfs_status dfs_plan_union_panel(const dfs_plan* plan, int layer, int which, cons
  * tables).  Host only. */
 dfs_status dfs_plan_memory(const dfs_plan* plan, int64_t* weight_bytes, int64_t* device_bytes);
 
-/* Algorithmic FLOPs (2 per multiply-add) of one block forward at (step, layer). */
+/* Algorithmic FLOPs (2 per multiply-add) of one block forward at (step, layer), closed
+ * form over the retained units only: 8 N dim head_dim h_s (QKV and output projections)
+ * + 4 N^2 head_dim h_s (Q K^T and P V) + 4 N dim f_s (FFN up and down), plus with
+ * cross-attention 4 N dim head_dim hc + 4 ctx_len dim head_dim hc + 4 N ctx_len head_dim hc;
+ * 0 for a block gated off.  The ratio to the keep-all value is the per-step FLOP
+ * retention that Sec. 5.4 reports (a 24% mean cut for Wan-14B) and Sec. 6 plots. */
 dfs_status dfs_plan_flops(const dfs_plan* plan, int step, int layer, double* flops);
 
 /* Workspace buffers left by the last forward on this plan (for intermediate checks):

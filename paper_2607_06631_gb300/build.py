@@ -2,12 +2,16 @@
 
 Every .cu translation unit under csrc/ is compiled in parallel with nvcc, then linked
 into paper_2607_06631_gb300/_lib/libdfs.so with the CUDA runtime linked statically.
-Objects go to _build/ at the repository root; both folders are git-ignored.
+Objects go to _build/ at the repository root; both folders are git-ignored.  A SHA-256
+fingerprint of the sources, header, flags, compiler version and machine type is stored
+beside the library, and the library is rebuilt whenever it differs.
 """
 from __future__ import annotations
 
 import concurrent.futures as cf
+import hashlib
 import os
+import platform
 import shutil
 import subprocess
 
@@ -17,9 +21,11 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIB_DIR, "libdfs.so")
+STAMP = LIB + ".sha256"
 BUILD = os.path.join(ROOT, "_build")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I" + INCLUDE]
+LINK = ["-shared", "-cudart", "static"]
 
 
 def _nvcc() -> str:
@@ -33,18 +39,36 @@ def sources():
     return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cu"))
 
 
-def _stale() -> bool:
-    if not os.path.exists(LIB):
-        return True
-    t = os.path.getmtime(LIB)
-    deps = sources() + [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cuh")]
+def _fingerprint() -> str:
+    """SHA-256 over every source the library is built from (the .cu / .cuh files and the
+    public header), the compiler flags, the nvcc version and the host machine type."""
+    h = hashlib.sha256()
+    deps = sorted(sources() + [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cuh")])
     deps.append(os.path.join(INCLUDE, "dfs.h"))
-    return any(os.path.getmtime(d) > t for d in deps)
+    for d in deps:
+        h.update(os.path.relpath(d, ROOT).encode())
+        with open(d, "rb") as f:
+            h.update(hashlib.sha256(f.read()).digest())
+    h.update(" ".join(ARCH + FLAGS[:-1] + LINK).encode())
+    r = subprocess.run([_nvcc(), "--version"], capture_output=True, text=True)
+    h.update(r.stdout.encode())
+    h.update(platform.machine().encode())
+    return h.hexdigest()
+
+
+def _stale(fp: str) -> bool:
+    """The library is rebuilt unless it exists and the fingerprint stored beside it at its
+    last build equals the current one (file times play no part)."""
+    if not (os.path.exists(LIB) and os.path.exists(STAMP)):
+        return True
+    with open(STAMP) as f:
+        return f.read().strip() != fp
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
     """Compiles (if needed) and returns the path of libdfs.so."""
-    if not force and not _stale():
+    fp = _fingerprint()
+    if not force and not _stale(fp):
         return LIB
     nvcc = _nvcc()
     os.makedirs(BUILD, exist_ok=True)
@@ -63,11 +87,13 @@ def build(force: bool = False, verbose: bool = False) -> str:
     with cf.ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
         objs = list(ex.map(compile_one, sources()))
     tmp = LIB + ".tmp"
-    cmd = [nvcc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs
+    cmd = [nvcc] + ARCH + LINK + ["-o", tmp] + objs
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError("link failed:\n%s%s" % (r.stdout, r.stderr))
     os.replace(tmp, LIB)
+    with open(STAMP, "w") as f:
+        f.write(fp + "\n")
     return LIB
 
 

@@ -917,6 +917,10 @@ dfs_status block_layer(dfs_plan* P, int step, int layer, const bf16* x, const bf
   return forward_impl(P, step, layer, x, out, st);
 }
 
+// Drops the cached device address of the allocation-free forward's static array for
+// `device` (defined with the array below).
+void noalloc_forget_device(int device);
+
 }  // namespace
 
 // ------------------------------------------------------------------ C ABI
@@ -946,6 +950,9 @@ dfs_status dfs_plan_create(const dfs_config* cfg, const dfs_layer_weights* layer
     free_plan(P);
     return e;
   }
+  // A plan exists only in a context created after the device's last reset, so the next
+  // allocation-free call looks the static array's address up again in this context.
+  noalloc_forget_device(P->device);
   *out = P;
   return DFS_OK;
 }
@@ -1358,8 +1365,17 @@ __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 std::mutex g_noalloc_mu;
 std::map<int, unsigned char*> g_noalloc_addr;  // device ordinal -> device address of the array
 
+void noalloc_forget_device(int device) {
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  g_noalloc_addr.erase(device);
+}
+
 // Looks up (once per device, with that device current) the device address of the
-// scratch array; host code cannot use the symbol itself as a device pointer.
+// scratch array; host code cannot use the symbol itself as a device pointer.  The cached
+// address is dropped whenever a plan is created on the device (dfs_plan_create), because
+// a device reset (cudaDeviceReset) reloads the module, possibly at another address, and
+// invalidates every plan made before it: any plan a later call can use was created after
+// the reset, and its creation cleared the entry.
 dfs_status noalloc_scratch(int device, unsigned char** out) {
   std::lock_guard<std::mutex> lock(g_noalloc_mu);
   auto it = g_noalloc_addr.find(device);
@@ -1404,6 +1420,8 @@ dfs_status noalloc_forward(dfs_plan* P, int s, int l, const bf16* x, const bf16*
                 off, kNoAllocScratchBytes);
   int dev = 0;
   DFS_CK(cudaGetDevice(&dev));
+  if (dev != P->device)
+    return fail(DFS_EINVAL, "the current device (%d) is not the plan's device (%d)", dev, P->device);
   unsigned char* base = nullptr;
   dfs_status e = noalloc_scratch(dev, &base);
   if (e) return e;

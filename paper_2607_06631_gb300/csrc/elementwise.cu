@@ -2,6 +2,8 @@
 // and affine LayerNorm (K2 / K7), QK RMSNorm + 3D RoPE (K3), the modulation GEMV (K6),
 // bias-only residual branches and the Euler update (K8).  All move 16-byte vectors and
 // reduce with warp shuffles.
+#include <atomic>
+
 #include "kernels.cuh"
 
 namespace dfs {
@@ -64,9 +66,11 @@ __global__ void gather_segs_kernel(bf16* __restrict__ dst, long long ld_dst, con
   }
 }
 
+// Grid-stride kernels get at most 16 CTAs per SM.
 int grid_for(long long work, int threads) {
   long long g = (work + threads - 1) / threads;
-  if (g > 152LL * 16) g = 152LL * 16;
+  const long long cap = 16LL * current_device_sms();
+  if (g > cap) g = cap;
   if (g < 1) g = 1;
   return static_cast<int>(g);
 }
@@ -448,6 +452,18 @@ cudaError_t launch_euler(bf16* x, const bf16* v, float dt, long long n, cudaStre
   const long long nvec = n / 8;
   euler_kernel<<<grid_for(nvec, 256), 256, 0, s>>>(x, v, dt, nvec);
   return cudaGetLastError();
+}
+
+int current_device_sms() {
+  constexpr int kMaxDevices = 64;
+  static std::atomic<int> cache[kMaxDevices];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 1;
+  int n = dev < kMaxDevices ? cache[dev].load(std::memory_order_relaxed) : 0;
+  if (n > 0) return n;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+  if (dev < kMaxDevices) cache[dev].store(n, std::memory_order_relaxed);
+  return n;
 }
 
 }  // namespace dfs

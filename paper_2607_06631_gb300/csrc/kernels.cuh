@@ -92,6 +92,9 @@ cudaError_t attention_prepare();
 
 // ------------------------------------------------------------------------ memory-bound kernels
 
+// Streaming multiprocessors of the current device (queried once per device, then cached).
+int current_device_sms();
+
 // K1: dst[i, :] = src[rows[i], :] for i < n_rows (cols elements, multiple of 8).
 cudaError_t launch_gather_rows(bf16* dst, long long ld_dst, const bf16* src, long long ld_src,
                                const int* rows, int n_rows, int cols, cudaStream_t s);

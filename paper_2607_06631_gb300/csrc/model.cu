@@ -103,7 +103,8 @@ __global__ void unpatchify_kernel(bf16* out, const bf16* base, const bf16* __res
 
 int blocks_for(long long work, int threads) {
   long long g = (work + threads - 1) / threads;
-  if (g > 152LL * 8) g = 152LL * 8;
+  const long long cap = 8LL * current_device_sms();
+  if (g > cap) g = cap;
   return static_cast<int>(g < 1 ? 1 : g);
 }
 
