@@ -71,3 +71,23 @@ def test_reference_arm_prints_one_contract_line_on_the_tiny_block():
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
     assert "512 query rows" in d["cpu_baseline"]["sample"]
+
+
+def test_cpu_baseline_slice_extrapolation_on_a_small_block():
+    """cpu_baseline times K / V over all N once (one query row) and a 512-row slice, and
+    extrapolates the block as T_KV + (N / 512) T_rows; a stack at that block's FLOP rate."""
+    import copy
+    import bench
+    cfg = synth.tiny(grid=(2, 16, 32))  # 1024 tokens: two slices' worth
+    cfg.name = "tiny_1024"
+    c = bench.cpu_baseline(cfg)
+    N = cfg.n_tokens
+    assert c["kind"] == "oracle" and c["value"] > 0 and c["slice_rows"] == 512
+    t = c["T_KV_s"] + (N / 512) * c["T_rows_s"]
+    assert abs(c["block_seconds_extrapolated"] - t) <= 0.02 + 1e-3 * t
+    assert "T = T_KV + (N / 512) T_rows" in c["formula"]
+    stack = copy.deepcopy(synth.tiny(n_layers=3))
+    s = bench.cpu_baseline(stack)
+    assert s["stack_seconds_extrapolated"] > 0
+    rate = s["block_flops"] / s["block_seconds_extrapolated"]
+    assert abs(s["stack_seconds_extrapolated"] - bench.stack_flops(stack) / rate) <= 0.1 + 1e-3 * s["stack_seconds_extrapolated"]

@@ -72,14 +72,19 @@ def test_wan14b_block_per_head_qk_norm():
 
 
 def test_wan14b_block_with_cross_attention():
-    errs = run_large(synth.wan14b_cross(), (0, 3), edge=32, spread=64)
+    """Every step: the self- and cross-attention head counts and the FFN width (its K tail)
+    differ per step."""
+    errs = run_large(synth.wan14b_cross(), range(4), edge=32, spread=64)
     for s, (e, b) in errs.items():
         assert e <= TOL and b <= TOL, (s, e, b)
 
 
-def test_720p_block_half_keep():
+def test_720p_block_every_keep_ratio():
+    """All six keep ratios of the 720p sweep (1.0 .. 0.5: 40 .. 20 heads, 13824 .. 6912 FFN
+    channels, so every step has its own attention grid and FFN K tail), on the first and
+    last 32 rows (75600 = 590*128 + 80: the last row tile is ragged) and 32 rows between."""
     cfg = synth.sweep720_all()
-    errs = run_large(cfg, (5,), edge=32, spread=64)  # step 5 keeps 20 heads / 6912 channels
+    errs = run_large(cfg, range(6), edge=32, spread=32)
     for s, (e, b) in errs.items():
         assert e <= TOL and b <= TOL, (s, e, b)
 
