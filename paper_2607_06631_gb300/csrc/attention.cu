@@ -13,14 +13,24 @@
 // issues  S0_j, PV1_{j-1}, S1_j, PV0_j, S0_{j+1}, PV1_j, ...  so either tile's softmax overlaps
 // two MMAs of the other tile; its commits are multicast to both CTAs' barriers.  Both CTAs'
 // TMA loads complete on the even CTA's barriers.  V arrives pre-transposed (V^T written by
-// the QKV projection's epilogue) so every shared-memory operand is K-major.  The running max
-// only moves when it grows by more than 2^8 (exact: the same stale max enters O and the row
-// sum); O is then rescaled in TMEM.
+// the QKV projection's epilogue) so every shared-memory operand is K-major.
+//
+// The softmax has no row-max pass after the first key block.  P of block j is taken with
+// the running offset m (the first block's exact row max, or a later one), which is exact for
+// any m because the numerator O and the row sum l share it; m only has to keep P finite and
+// representable.  A row whose block sum stays within kSumLimit has every P of the block
+// within it; otherwise (or for a non-finite sum) the warp redoes the block with the exact
+// maximum and rescales O (in TMEM) and l.  So the exponentials start as soon as S is in
+// registers, and a tile's softmax is one pass: TMEM load, exponentials and packing, P store.
 //
 //   warp 0      TMA: own Q0, Q1 once; own halves of K_j and V^T_j into three-deep rings
 //   warp 1      TMEM allocation (collective over the pair); in the even CTA also the MMA thread
-//   warps 2..5  softmax / rescale / output of tile 0
-//   warps 6..9  softmax / rescale / output of tile 1
+//   warps 2..3  idle (they complete warpgroup 0, whose registers go to the softmax warpgroups)
+//   warps 4..7  softmax / rescale / output of tile 0
+//   warps 8..11 softmax / rescale / output of tile 1
+// The warpgroups split the register file unevenly (setmaxnreg): 88 registers per thread in
+// warpgroup 0, 208 in the softmax warpgroups, which then hold a row's 128 scores and its
+// packed P without spilling to local memory.
 #include "kernels.cuh"
 
 namespace dfs {
@@ -29,8 +39,30 @@ namespace {
 constexpr int kBM = 128;   // query rows per tile (two tiles per CTA, four per pair)
 constexpr int kBN = 128;   // key / value rows per block
 constexpr int kStages = 3; // K and V ring depth
-constexpr int kThreads = 320;
-constexpr float kRescaleThreshold = 8.f;  // log2 units
+constexpr int kThreads = 384;
+// Register split between the warpgroups (setmaxnreg): the launch gives every thread
+// kRegsLaunch registers (384 threads x 168 = 64512 of the SM's 65536; ptxas reports 168 for
+// this kernel); the TMA / MMA warpgroup gives part of its share to the two softmax
+// warpgroups.  The shares add up to the launch's total, 128 x 88 + 256 x 208 = 384 x 168,
+// and per SM sub-partition (one warp of each warpgroup) 88 + 208 + 208 = 504 registers x 32
+// lanes <= its 16384.  A larger softmax share would make the increase wait forever.
+constexpr int kRegsLaunch = 168, kRegsControl = 88, kRegsSoftmax = 208;
+static_assert(128 * kRegsControl + 256 * kRegsSoftmax <= kThreads * kRegsLaunch, "register split exceeds the launch");
+static_assert(kThreads * kRegsLaunch <= 65536, "launch registers exceed the SM");
+static_assert((kRegsControl + 2 * kRegsSoftmax) * 32 <= 16384, "register split exceeds a sub-partition");
+// Largest accepted row sum of one key block's P (every P of such a row is at most this):
+// far from fp32 / bf16 overflow, so O and l accumulate safely with a stale offset.
+constexpr float kSumLimit = 65536.f;
+
+// Store of 32 consecutive 32-bit TMEM columns without the wait (tcgen05.wait::st follows later).
+__device__ __forceinline__ void tmem_st32u_async(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n"
+      ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 template <int DH>
 struct AttnLayout {
@@ -101,119 +133,124 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   bool failed = false;
 
-  if (warp == 0) {
-    if (lane == 0) {
-      tma_prefetch_desc(&p.tma_q);
-      tma_prefetch_desc(&p.tma_k);
-      tma_prefetch_desc(&p.tma_vt);
-      const int qx = p.q_col0 + head * DH;
-      const int kx = p.k_col0 + head * DH;
-      const uint32_t lq = map_to_rank(q_full, 0);
-      if (rank == 0) mbar_arrive_expect_tx(q_full, 2 * 2 * L::kQBytes);
+  if (warp < 4) {
+    // warpgroup 0 (TMA, MMA, two idle warps) hands registers to the softmax warpgroups
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsControl));
+    if (warp == 0) {
+      if (lane == 0) {
+        tma_prefetch_desc(&p.tma_q);
+        tma_prefetch_desc(&p.tma_k);
+        tma_prefetch_desc(&p.tma_vt);
+        const int qx = p.q_col0 + head * DH;
+        const int kx = p.k_col0 + head * DH;
+        const uint32_t lq = map_to_rank(q_full, 0);
+        if (rank == 0) mbar_arrive_expect_tx(q_full, 2 * 2 * L::kQBytes);
 #pragma unroll
-      for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int c = 0; c < DH / 64; ++c)
-          tma_load_2d_pair(sQ + i * L::kQBytes + c * (kBM * 128), &p.tma_q, lq, qx + 64 * c, q_base + i * kBM);
-      // K runs one block ahead of V: K_j is needed by S0_j long before V_j by PV0_j
-      for (int j = 0; j <= nkv && !failed; ++j) {
-        if (j < nkv) {
-          const int s = j % kStages;
-          if (!mbar_wait_cluster(&k_empty[s], ((j / kStages) & 1) ^ 1, p.err)) { failed = true; break; }
-          if (rank == 0) mbar_arrive_expect_tx(&k_full[s], 2 * L::kKBytes);
-          const uint32_t lk = map_to_rank(&k_full[s], 0);
+        for (int i = 0; i < 2; ++i)
 #pragma unroll
           for (int c = 0; c < DH / 64; ++c)
-            tma_load_2d_pair(sK + s * L::kKBytes + c * L::kKPanel, &p.tma_k, lk, kx + 64 * c,
-                             j * kBN + static_cast<int>(rank) * (kBN / 2));
-        }
-        if (j >= 1) {
-          const int jv = j - 1, s = jv % kStages;
-          if (!mbar_wait_cluster(&v_empty[s], ((jv / kStages) & 1) ^ 1, p.err)) { failed = true; break; }
-          if (rank == 0) mbar_arrive_expect_tx(&v_full[s], 2 * L::kVBytes);
-          const uint32_t lv = map_to_rank(&v_full[s], 0);
+            tma_load_2d_pair(sQ + i * L::kQBytes + c * (kBM * 128), &p.tma_q, lq, qx + 64 * c, q_base + i * kBM);
+        // K runs one block ahead of V: K_j is needed by S0_j long before V_j by PV0_j
+        for (int j = 0; j <= nkv && !failed; ++j) {
+          if (j < nkv) {
+            const int s = j % kStages;
+            if (!mbar_wait_cluster(&k_empty[s], ((j / kStages) & 1) ^ 1, p.err)) { failed = true; break; }
+            if (rank == 0) mbar_arrive_expect_tx(&k_full[s], 2 * L::kKBytes);
+            const uint32_t lk = map_to_rank(&k_full[s], 0);
 #pragma unroll
-          for (int c = 0; c < kBN / 64; ++c)
-            tma_load_2d_pair(sV + s * L::kVBytes + c * L::kVPanel, &p.tma_vt, lv, jv * kBN + 64 * c,
-                             head * DH + static_cast<int>(rank) * (DH / 2));
+            for (int c = 0; c < DH / 64; ++c)
+              tma_load_2d_pair(sK + s * L::kKBytes + c * L::kKPanel, &p.tma_k, lk, kx + 64 * c,
+                               j * kBN + static_cast<int>(rank) * (kBN / 2));
+          }
+          if (j >= 1) {
+            const int jv = j - 1, s = jv % kStages;
+            if (!mbar_wait_cluster(&v_empty[s], ((jv / kStages) & 1) ^ 1, p.err)) { failed = true; break; }
+            if (rank == 0) mbar_arrive_expect_tx(&v_full[s], 2 * L::kVBytes);
+            const uint32_t lv = map_to_rank(&v_full[s], 0);
+#pragma unroll
+            for (int c = 0; c < kBN / 64; ++c)
+              tma_load_2d_pair(sV + s * L::kVBytes + c * L::kVPanel, &p.tma_vt, lv, jv * kBN + 64 * c,
+                               head * DH + static_cast<int>(rank) * (DH / 2));
+          }
         }
       }
-    }
-  } else if (warp == 1) {
-    if (lane == 0 && rank == 0) {
-      constexpr uint32_t idesc_s = idesc_bf16(2 * kBM, kBN);
-      constexpr uint32_t idesc_o = idesc_bf16(2 * kBM, DH);
-      // Descriptors are built once: the issue loop only adds constant offsets (the start
-      // address field holds address >> 4), which keeps this thread's issue rate at the
-      // tensor pipe's rate.
-      const uint64_t dq = sw128_desc(smem_u32(sQ));
-      const uint64_t dk = sw128_desc(smem_u32(sK));
-      const uint64_t dv = sw128_desc(smem_u32(sV));
-      // S_i(j) = Q_i K_j^T into S_i's TMEM columns of both CTAs
-      auto issue_s = [&](int i, int j) {
-        const uint64_t a = dq + static_cast<uint64_t>(i * (L::kQBytes >> 4));
-        const uint64_t b = dk + static_cast<uint64_t>((j % kStages) * (L::kKBytes >> 4));
-        const uint32_t d = tmem + i * kBN;
+    } else if (warp == 1) {
+      if (lane == 0 && rank == 0) {
+        constexpr uint32_t idesc_s = idesc_bf16(2 * kBM, kBN);
+        constexpr uint32_t idesc_o = idesc_bf16(2 * kBM, DH);
+        // Descriptors are built once: the issue loop only adds constant offsets (the start
+        // address field holds address >> 4), which keeps this thread's issue rate at the
+        // tensor pipe's rate.
+        const uint64_t dq = sw128_desc(smem_u32(sQ));
+        const uint64_t dk = sw128_desc(smem_u32(sK));
+        const uint64_t dv = sw128_desc(smem_u32(sV));
+        // S_i(j) = Q_i K_j^T into S_i's TMEM columns of both CTAs
+        auto issue_s = [&](int i, int j) {
+          const uint64_t a = dq + static_cast<uint64_t>(i * (L::kQBytes >> 4));
+          const uint64_t b = dk + static_cast<uint64_t>((j % kStages) * (L::kKBytes >> 4));
+          const uint32_t d = tmem + i * kBN;
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          constexpr uint32_t qpanel = (kBM * 128) >> 4, kpanel = L::kKPanel >> 4;
-          mma_pair_ss(d, a + (kk / 4) * qpanel + (kk % 4) * 2, b + (kk / 4) * kpanel + (kk % 4) * 2, idesc_s,
-                      kk != 0);
-        }
-        commit_pair(&s_full[i]);
-      };
-      // O_i += P_i(j) V_j with P_i read from the first 64 columns of S_i in both CTAs
-      auto issue_pv = [&](int i, int j) {
-        const uint64_t b = dv + static_cast<uint64_t>((j % kStages) * (L::kVBytes >> 4));
-        const uint32_t d = tmem + 256 + i * 128, a = tmem + i * kBN;
-        const uint32_t first = j != 0;
-#pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
-          constexpr uint32_t vpanel = L::kVPanel >> 4;
-          mma_pair_ts(d, a + kk * 8, b + (kk / 4) * vpanel + (kk % 4) * 2, idesc_o, kk == 0 ? first : 1u);
-        }
-      };
-      do {
-        if (!mbar_wait_cluster(q_full, 0, p.err)) { failed = true; break; }
-        if (!mbar_wait_cluster(&k_full[0], 0, p.err)) { failed = true; break; }
-        tc_fence_after();
-        issue_s(0, 0);
-        issue_s(1, 0);
-        commit_pair(&k_empty[0]);
-        for (int j = 0; j < nkv; ++j) {
-          const int s = j % kStages;
-          const uint32_t ph = (j / kStages) & 1;
-          // PV0_j
-          if (!mbar_wait_cluster(&p_full[0], j & 1, p.err) || !mbar_wait_cluster(&v_full[s], ph, p.err)) {
-            failed = true;
-            break;
+          for (int kk = 0; kk < DH / 16; ++kk) {
+            constexpr uint32_t qpanel = (kBM * 128) >> 4, kpanel = L::kKPanel >> 4;
+            mma_pair_ss(d, a + (kk / 4) * qpanel + (kk % 4) * 2, b + (kk / 4) * kpanel + (kk % 4) * 2, idesc_s,
+                        kk != 0);
           }
+          commit_pair(&s_full[i]);
+        };
+        // O_i += P_i(j) V_j with P_i read from the first 64 columns of S_i in both CTAs
+        auto issue_pv = [&](int i, int j) {
+          const uint64_t b = dv + static_cast<uint64_t>((j % kStages) * (L::kVBytes >> 4));
+          const uint32_t d = tmem + 256 + i * 128, a = tmem + i * kBN;
+          const uint32_t first = j != 0;
+#pragma unroll
+          for (int kk = 0; kk < kBN / 16; ++kk) {
+            constexpr uint32_t vpanel = L::kVPanel >> 4;
+            mma_pair_ts(d, a + kk * 8, b + (kk / 4) * vpanel + (kk % 4) * 2, idesc_o, kk == 0 ? first : 1u);
+          }
+        };
+        do {
+          if (!mbar_wait_cluster(q_full, 0, p.err)) { failed = true; break; }
+          if (!mbar_wait_cluster(&k_full[0], 0, p.err)) { failed = true; break; }
           tc_fence_after();
-          issue_pv(0, j);
-          if (j + 1 == nkv) commit_pair(&o_done[0]);
-          // S0_{j+1}
-          if (j + 1 < nkv) {
-            const int s1 = (j + 1) % kStages;
-            if (!mbar_wait_cluster(&k_full[s1], ((j + 1) / kStages) & 1, p.err)) { failed = true; break; }
+          issue_s(0, 0);
+          issue_s(1, 0);
+          commit_pair(&k_empty[0]);
+          for (int j = 0; j < nkv; ++j) {
+            const int s = j % kStages;
+            const uint32_t ph = (j / kStages) & 1;
+            // PV0_j
+            if (!mbar_wait_cluster(&p_full[0], j & 1, p.err) || !mbar_wait_cluster(&v_full[s], ph, p.err)) {
+              failed = true;
+              break;
+            }
             tc_fence_after();
-            issue_s(0, j + 1);
+            issue_pv(0, j);
+            if (j + 1 == nkv) commit_pair(&o_done[0]);
+            // S0_{j+1}
+            if (j + 1 < nkv) {
+              const int s1 = (j + 1) % kStages;
+              if (!mbar_wait_cluster(&k_full[s1], ((j + 1) / kStages) & 1, p.err)) { failed = true; break; }
+              tc_fence_after();
+              issue_s(0, j + 1);
+            }
+            // PV1_j
+            if (!mbar_wait_cluster(&p_full[1], j & 1, p.err)) { failed = true; break; }
+            tc_fence_after();
+            issue_pv(1, j);
+            commit_pair(&v_empty[s]);
+            if (j + 1 == nkv) commit_pair(&o_done[1]);
+            // S1_{j+1}
+            if (j + 1 < nkv) {
+              issue_s(1, j + 1);
+              commit_pair(&k_empty[(j + 1) % kStages]);
+            }
           }
-          // PV1_j
-          if (!mbar_wait_cluster(&p_full[1], j & 1, p.err)) { failed = true; break; }
-          tc_fence_after();
-          issue_pv(1, j);
-          commit_pair(&v_empty[s]);
-          if (j + 1 == nkv) commit_pair(&o_done[1]);
-          // S1_{j+1}
-          if (j + 1 < nkv) {
-            issue_s(1, j + 1);
-            commit_pair(&k_empty[(j + 1) % kStages]);
-          }
-        }
-      } while (false);
+        } while (false);
+      }
     }
   } else {
-    const int tile = (warp - 2) >> 2;        // 0: warps 2..5, 1: warps 6..9
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsSoftmax));
+    const int tile = (warp - 4) >> 2;        // 0: warps 4..7, 1: warps 8..11
     const int sub = warp & 3;                // TMEM lane quarter this warp may access
     const int r = sub * 32 + lane;           // query row within the tile = TMEM lane
     const uint32_t lane_addr = static_cast<uint32_t>(sub * 32) << 16;
@@ -222,7 +259,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int q_row = q_base + tile * kBM + r;
     const uint32_t p_full_leader = map_to_rank(&p_full[tile], 0);
     const float sl2 = p.scale_log2;
-    float m_run = -INFINITY;                 // running max of the scaled scores (log2 units)
+    float m_run = -INFINITY;                 // offset of P (log2 units): block 0's row max, raised by redone blocks
     float l_run = 0.f;
     for (int j = 0; j < nkv; ++j) {
       const bool ok = mbar_wait_cluster(&s_full[tile], j & 1, p.err);
@@ -236,23 +273,55 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int i = 0; i < kBN; ++i)
           if (i >= valid) s[i] = -INFINITY;
       }
-      // row max: 8 independent chains of three-input maxima
-      float pm[8];
+      // row max of the scaled scores: 8 independent chains of three-input maxima
+      auto row_max = [&]() {
+        float pm[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) pm[i] = s[i];
+        for (int i = 0; i < 8; ++i) pm[i] = s[i];
 #pragma unroll
-      for (int i = 8; i < kBN; i += 16)
+        for (int i = 8; i < kBN; i += 16)
 #pragma unroll
-        for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
-      const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])) * sl2;
-      const bool move = mx > m_run + kRescaleThreshold;
-      if (j == 0) {
-        m_run = mx;
-      } else if (__any_sync(0xffffffffu, move)) {
-        // S_i(j) completing implies P_i(j-1) V_{j-1} completed: O_i is stable here
-        const float alpha = move ? fast_exp2(m_run - mx) : 1.f;
-        if (move) m_run = mx;
+          for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
+        return fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])) * sl2;
+      };
+      // P = exp2(s * scale - m_run) as bf16 pairs into the first 64 columns of S_i (the first
+      // half's store overlaps the second half's arithmetic); returns the block's row sum.
+      // Scale-and-shift and the row-sum partials run as packed pairs.
+      auto write_p = [&]() {
+        const float neg_m = -m_run;
+        float ps[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) ps[i] = 0.f;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            float x0, x1;
+            ffma2(x0, x1, s[64 * h + 2 * c], s[64 * h + 2 * c + 1], sl2, sl2, neg_m, neg_m);
+            const float e0 = fast_exp2(x0);
+            const float e1 = fast_exp2(x1);
+            fadd2(ps[2 * (c & 3)], ps[2 * (c & 3) + 1], e0, e1);
+            pk[c] = pack_bf16x2(e0, e1);
+          }
+          tmem_st32u_async(tS + 32 * h, pk);
+        }
+        tmem_wait_st();
+        return ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+      };
+      // The first block sets the running max exactly.  Later blocks reuse it without a max
+      // pass: their P are exact for any offset (numerator and row sum share it), and only
+      // their size matters.  A block row sum within kSumLimit bounds every P of that row by
+      // it; a larger (or non-finite) sum in any row of the warp makes the warp redo the block
+      // with the exact maximum, rescaling O and the row sum.
+      if (j == 0) m_run = row_max();
+      float l_blk = write_p();
+      if (__any_sync(0xffffffffu, !(l_blk <= kSumLimit))) {
+        const float m_new = fmaxf(m_run, row_max());
+        const float alpha = fast_exp2(m_run - m_new);
+        m_run = m_new;
         l_run *= alpha;
+        // S_i(j) completing implies P_i(j-1) V_{j-1} completed: O_i is stable here
 #pragma unroll
         for (int c = 0; c < DH / 32; ++c) {
           float o[32];
@@ -261,28 +330,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           for (int i = 0; i < 32; ++i) o[i] *= alpha;
           tmem_st32(tO + 32 * c, o);
         }
+        l_blk = write_p();
       }
-      // P = exp2(s * scale - m_run) as bf16 pairs into the first 64 columns of S_i;
-      // scale-and-shift and the row-sum partials run as packed pairs
-      const float neg_m = -m_run;
-      float ps[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ps[i] = 0.f;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        uint32_t pk[32];
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          float x0, x1;
-          ffma2(x0, x1, s[64 * h + 2 * c], s[64 * h + 2 * c + 1], sl2, sl2, neg_m, neg_m);
-          const float e0 = fast_exp2(x0);
-          const float e1 = fast_exp2(x1);
-          fadd2(ps[2 * (c & 3)], ps[2 * (c & 3) + 1], e0, e1);
-          pk[c] = pack_bf16x2(e0, e1);
-        }
-        tmem_st32u(tS + 32 * h, pk);
-      }
-      l_run += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+      l_run += l_blk;
       // The TMEM stores of P are complete (tcgen05.wait::st) and ordered before this
       // thread-sync point by the tcgen05 fence; the MMA thread orders its MMAs after its
       // wait with tcgen05.fence::after_thread_sync.  One arrival per warp: local in the
