@@ -315,13 +315,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       // it; a larger (or non-finite) sum in any row of the warp makes the warp redo the block
       // with the exact maximum, rescaling O and the row sum.
       if (j == 0) m_run = row_max();
-      float l_blk = write_p();
-      if (__any_sync(0xffffffffu, !(l_blk <= kSumLimit))) {
+      float l_blk, alpha = 1.f;
+      for (int pass = 0;; ++pass) {
+        l_blk = write_p();
+        if (pass == 1 || !__any_sync(0xffffffffu, !(l_blk <= kSumLimit))) break;
         const float m_new = fmaxf(m_run, row_max());
-        const float alpha = fast_exp2(m_run - m_new);
+        alpha = fast_exp2(m_run - m_new);
         m_run = m_new;
+      }
+      if (__any_sync(0xffffffffu, alpha != 1.f)) {
+        // S_i(j) completing implies P_i(j-1) V_{j-1} completed: O_i is stable here, and
+        // P_i(j) V_j is issued only after this warp's arrival below
         l_run *= alpha;
-        // S_i(j) completing implies P_i(j-1) V_{j-1} completed: O_i is stable here
 #pragma unroll
         for (int c = 0; c < DH / 32; ++c) {
           float o[32];
@@ -330,7 +335,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           for (int i = 0; i < 32; ++i) o[i] *= alpha;
           tmem_st32(tO + 32 * c, o);
         }
-        l_blk = write_p();
       }
       l_run += l_blk;
       // The TMEM stores of P are complete (tcgen05.wait::st) and ordered before this
