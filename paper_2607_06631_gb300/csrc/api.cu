@@ -368,6 +368,7 @@ dfs::GemmArgs gemm_args(dfs_plan* P, const CUtensorMap& a, const CUtensorMap& b,
   g.bias = bias;
   g.split = N;
   g.group = dfs::gemm_group(K);
+  g.epi_warps = dfs::gemm_epilogue_warps(K);
   g.err = P->err;
   return g;
 }

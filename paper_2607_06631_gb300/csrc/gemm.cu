@@ -13,11 +13,16 @@
 //   warp 1      TMEM allocation (collective over the pair); in the even CTA the MMA thread,
 //               issuing into one of two accumulators (2 x 256 fp32 columns per CTA), so the
 //               epilogue of tile i overlaps the main loop of tile i+1.
-//   warps 2..5  epilogue of this CTA's 128 rows: tcgen05.ld 32 columns at a time, fused bias /
+//   warps 2..3  idle (they complete warpgroup 0, whose registers go to the epilogue warpgroups)
+//   warps 4..11 epilogue of this CTA's 128 rows: tcgen05.ld 32 columns at a time, fused bias /
 //               GELU / gated residual, predicated stores for the ragged M and N edges.  A
 //               thread owns one output row, so every global access of a warp touches 32 rows;
 //               where bases and row pitches allow, the accesses are 256-bit (one full 32-byte
 //               sector per row per instruction) to halve the number of L1 / L2 transactions.
+//               Short reductions use all 8 warps (two per TMEM lane quarter, 128 columns each),
+//               long ones warps 4..7 only (GemmArgs::epi_warps).
+// setmaxnreg splits the registers: 72 per thread in warpgroup 0, 216 in the epilogue
+// warpgroups (launch 384 x 168 = 128 x 72 + 256 x 216).
 // Ragged K (f_s is a multiple of 8, not of 64) is covered by TMA zero fill.
 #include "kernels.cuh"
 
@@ -33,7 +38,8 @@ __device__ __forceinline__ float gelu_tanh(float x) {
 }
 
 // Grouped raster: G M-tiles share each sweep over N so that concurrent CTA pairs reuse both
-// operands from L2.
+// operands from L2; the sweep direction alternates between groups (serpentine), so each group
+// starts on the B bands its predecessor finished with.
 __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int G, int& mt, int& nt) {
   const int group = tile / (G * n_tiles);
   const int first_m = group * G;
@@ -41,6 +47,7 @@ __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, 
   const int local = tile - group * G * n_tiles;
   mt = first_m + local % gsz;
   nt = local / gsz;
+  if (group & 1) nt = n_tiles - 1 - nt;
 }
 
 __device__ __forceinline__ void st_global_32B(void* dst, const uint4& a, const uint4& b);
@@ -203,6 +210,7 @@ __device__ __forceinline__ void load_res_chunk(int res_f32, const char* rrow, in
 // flight instead of waiting out one memory latency per 32 columns.  The residual may be the
 // output itself (in-place update): every element is still read by its own thread before
 // that thread writes it.
+template <int NCH>
 __device__ __forceinline__ void epilogue_gated_row(const GemmArgs& p, int row, int colb, uint32_t taddr) {
   const char* rrow = static_cast<const char*>(p.res) +
                      (static_cast<long long>(row) * p.ldr + colb) * (p.res_f32 ? 4 : 2);
@@ -210,8 +218,8 @@ __device__ __forceinline__ void epilogue_gated_row(const GemmArgs& p, int row, i
   load_res_chunk(p.res_f32, rrow, 0, w[0]);
   load_res_chunk(p.res_f32, rrow, 1, w[1]);
 #pragma unroll
-  for (int c = 0; c < kGemmBN / 32; ++c) {
-    if (c + 2 < kGemmBN / 32) load_res_chunk(p.res_f32, rrow, c + 2, w[(c + 2) % 3]);
+  for (int c = 0; c < NCH; ++c) {
+    if (c + 2 < NCH) load_res_chunk(p.res_f32, rrow, c + 2, w[(c + 2) % 3]);
     const int col0 = colb + 32 * c;
     float v[32];
     tmem_ld32(taddr + 32 * c, v);
@@ -309,7 +317,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 8);  // one arrival per epilogue warp of the pair
+      mbar_init(&tempty[a], 2 * p.epi_warps);  // one arrival per epilogue warp of the pair
     }
     fence_mbar_init();
   }
@@ -326,6 +334,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
   bool failed = false;
 
+  if (warp < 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kGemmRegsControl));
   if (warp == 0) {
     if (lane == 0 && kb > 0) {
       tma_prefetch_desc(&p.tma_a);
@@ -398,8 +408,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         if (acc == 0) acc_phase ^= 1;
       }
     }
+  }
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kGemmRegsEpilogue));
     const int sub = warp & 3;  // TMEM lane quarter this warp may access
+    // with 8 epilogue warps each lane quarter's two warps take 128 columns of every tile; with
+    // 4, warps 4..7 take all 256 and warps 8..11 have no work
+    const int half = (warp - 4) >> 2;
+    const int c_lo = p.epi_warps == 8 ? 128 * half : 0, c_n = p.epi_warps == 8 ? 128 : kGemmBN;
+    const bool idle = p.epi_warps != 8 && half == 1;
     const int r_in_tile = static_cast<int>(rank) * kGemmBM + sub * 32 + lane;
     // the wide epilogue reads and writes 32-byte pieces: bases and row pitches must keep them aligned
     const int osz = p.out_f32 ? 4 : 2, rsz = p.res_f32 ? 4 : 2;
@@ -409,7 +426,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     const uint32_t tempty_leader0 = map_to_rank(&tempty[0], 0), tempty_leader1 = map_to_rank(&tempty[1], 0);
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = pair; tile < num_tiles; tile += n_pairs) {
+    for (int tile = pair; tile < num_tiles && !idle; tile += n_pairs) {
       int mt, nt;
       tile_coords(tile, m_tiles, n_tiles, p.group, mt, nt);
       const int row = mt * kGemmTileM + r_in_tile;
@@ -422,11 +439,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       }
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * kGemmBN;
       // warp-uniform choice: the TMEM loads on both paths are warp-collective
-      if (p.mode == kEpiGatedRes && kb > 0 && (nt + 1) * kGemmBN <= p.N && wide_ok &&
+      if (p.mode == kEpiGatedRes && kb > 0 && nt * kGemmBN + c_lo + c_n <= p.N && wide_ok &&
           __all_sync(0xffffffffu, row < p.M)) {
-        epilogue_gated_row(p, row, nt * kGemmBN, tacc);
+        for (int c = c_lo; c < c_lo + c_n; c += 128) epilogue_gated_row<4>(p, row, nt * kGemmBN + c, tacc + c);
       } else {
-        for (int c = 0; c < kGemmBN; c += 32) {
+        for (int c = c_lo; c < c_lo + c_n; c += 32) {
           const int col0 = nt * kGemmBN + c;
           if (col0 >= p.N) break;
           float v[32];
@@ -477,6 +494,7 @@ cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t s) {
   const int tiles = m_tiles * n_tiles;
   if (tiles == 0) return cudaSuccess;
   const int pairs = tiles < num_sms / 2 ? tiles : num_sms / 2;
+  if (a.epi_warps != 4 && a.epi_warps != 8) return cudaErrorInvalidValue;
   gemm_bf16_tcgen05<<<2 * pairs, kGemmThreads, kGemmSmem, s>>>(a);
   return cudaGetLastError();
 }

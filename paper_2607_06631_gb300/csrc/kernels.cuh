@@ -18,7 +18,12 @@ enum EpiMode : int {
 // A CTA pair computes a kGemmTileM x kGemmBN output tile; each CTA stages kGemmBM rows of A
 // and kGemmBRows rows of B per K block.
 constexpr int kGemmBM = 128, kGemmTileM = 256, kGemmBN = 256, kGemmBRows = 128, kGemmBK = 64, kGemmStages = 6;
-constexpr int kGemmThreads = 192;
+constexpr int kGemmThreads = 384;  // warpgroup 0: TMA, MMA, 2 idle warps; warpgroups 1-2: epilogue
+// Register split (setmaxnreg) between warpgroup 0 and the two epilogue warpgroups; launch
+// 384 x 168 registers; 128 x kGemmRegsControl + 256 x kGemmRegsEpilogue must not exceed it.
+constexpr int kGemmRegsLaunch = 168, kGemmRegsControl = 72, kGemmRegsEpilogue = 216;
+static_assert(128 * kGemmRegsControl + 256 * kGemmRegsEpilogue <= kGemmThreads * kGemmRegsLaunch, "GEMM register split exceeds the launch");
+static_assert((kGemmRegsControl + 2 * kGemmRegsEpilogue) * 32 <= 16384, "GEMM register split exceeds a sub-partition");
 constexpr int kGemmABytes = kGemmBM * kGemmBK * 2;
 constexpr int kGemmBBytes = kGemmBRows * kGemmBK * 2;
 constexpr int kGemmStageBytes = kGemmABytes + kGemmBBytes;
@@ -56,7 +61,9 @@ struct GemmArgs {
   long long ldr;
   int res_f32;
   const float* gate;  // [N] or null (gate = 1)
-  int group;          // M tiles per raster group (tiles of one group sweep N together)
+  int epi_warps;      // epilogue warps per CTA: 8 (two per TMEM lane quarter, 128 columns each) or 4
+  int group;          // M tiles per raster group (tiles of one group sweep N together; odd groups
+                      // sweep N backwards, so a group starts on the B bands the previous one ended on)
   int b_gather;       // GatherMode
   int b_group;        // kGatherRows: rows per group (64 or 128)
   unsigned short b_idx[kGemmMapMax];  // index map of the gather (see GatherMode)
@@ -64,13 +71,18 @@ struct GemmArgs {
 };
 
 cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t s);
-// M tiles per raster group for a reduction length K.  On the Wan-14B-shaped block (K = 5120
-// and 13824) groups of 16 tiles were as fast as 8 or a K-dependent size that keeps one group's
-// A rows within 40 MB of L2, and 1-5% faster than 4: the GEMMs are not limited by re-reads.
-inline int gemm_group(int K) {
-  (void)K;
-  return 16;
-}
+// M tiles per raster group for a reduction length K: 16 up to K = 6144, 8 beyond.  A group's
+// A bands (256 rows x K each) stay in L2 while its tiles sweep N; with the long reductions of
+// the FFN down projection (K = f_s up to 13824, 7 MB per band) 16 bands crowd out the B bands
+// that the concurrent tiles share.  Measured on the Wan-14B-shaped down projections (GB300,
+// serpentine order): groups of 8 ran 4% faster than 16 at 75600 tokens and 1.5% at 32760;
+// 4, 6, 12 and 24 were slower; for K = 5120 (QKV, FFN up) 16 was fastest.
+inline int gemm_group(int K) { return K > 6144 ? 8 : 16; }
+// Epilogue warps per CTA for a reduction length K: with short reductions (K <= 2048, e.g. the
+// Wan-1.3B-shaped projections at K = 1536) a tile's main loop is shorter than its epilogue,
+// which 8 warps run in about half the time; with long ones 4 warps leave more of the memory
+// system to the main loop.
+inline int gemm_epilogue_warps(int K) { return K <= 2048 ? 8 : 4; }
 cudaError_t gemm_prepare();  // opts the kernel into its shared-memory size
 
 // ------------------------------------------------------------------------ K5 attention
