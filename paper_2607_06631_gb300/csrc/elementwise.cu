@@ -40,6 +40,30 @@ __device__ __forceinline__ float2 block_sum2(float a, float b, float (*red)[32])
   return make_float2(warp_sum(l < nw ? red[0][l] : 0.f), warp_sum(l < nw ? red[1][l] : 0.f));
 }
 
+// Two sums over each group of TPR consecutive threads (TPR a multiple of 32 dividing blockDim.x),
+// every thread getting its group's sums.  Its two barriers involve the whole CTA.
+template <int TPR>
+__device__ __forceinline__ float2 group_sum2(float a, float b, float (*red)[32]) {
+  a = warp_sum(a);
+  b = warp_sum(b);
+  constexpr int kWarps = TPR / 32;
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) {
+    red[0][w] = a;
+    red[1][w] = b;
+  }
+  __syncthreads();
+  const int g0 = (w / kWarps) * kWarps;
+  float ta = 0.f, tb = 0.f;
+#pragma unroll
+  for (int i = 0; i < kWarps; ++i) {
+    ta += red[0][g0 + i];
+    tb += red[1][g0 + i];
+  }
+  return make_float2(ta, tb);
+}
+
 // ------------------------------------------------------------------ K1 compaction
 
 __global__ void gather_rows_kernel(bf16* __restrict__ dst, long long ld_dst, const bf16* __restrict__ src,
@@ -85,12 +109,28 @@ __global__ void modulation_kernel(float* __restrict__ out, const bf16* __restric
   const uint4* w4 = reinterpret_cast<const uint4*>(W + static_cast<long long>(warp) * cols);
   const uint4* t4 = reinterpret_cast<const uint4*>(t);
   float acc = 0.f;
-  for (int v = lane; v < cols / 8; v += 32) {
-    float a[8], x[8];
-    unpack_bf16x8(__ldg(w4 + v), a);
-    unpack_bf16x8(__ldg(t4 + v), x);
+  const int nv = cols / 8;
+  // four 16-byte loads of W in flight per lane before their products are accumulated
+  for (int v0 = lane; v0 < nv; v0 += 4 * 32) {
+    uint4 wv[4], tv[4];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) acc = fmaf(a[i], x[i], acc);
+    for (int u = 0; u < 4; ++u) {
+      const int v = v0 + 32 * u;
+      if (v < nv) {
+        wv[u] = __ldg(w4 + v);
+        tv[u] = __ldg(t4 + v);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (v0 + 32 * u < nv) {
+        float a[8], x[8];
+        unpack_bf16x8(wv[u], a);
+        unpack_bf16x8(tv[u], x);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc = fmaf(a[i], x[i], acc);
+      }
+    }
   }
   acc = warp_sum(acc);
   if (lane == 0) {
@@ -108,12 +148,12 @@ __global__ void add_table_kernel(float* out, const float* base, const bf16* e, i
 // ------------------------------------------------------------------ K2 / K7 row LayerNorm
 
 
-// One CTA of NT threads per row with the row held in registers (VPT 8-wide vectors per thread;
-// 128 threads and 8 CTAs per SM up to 5120 columns, 256 threads beyond): the row is read from
-// memory once.  Mean and variance come from one
-// CTA reduction of two sums in the shifted-data form: sums of x - K and (x - K)^2 with K the
-// row's first element, which keeps E[(x-K)^2] - E[x-K]^2 free of cancellation however large
-// the row's mean.
+// A group of TPR threads per row, 256 / TPR rows per CTA (4 CTAs of 256 threads per SM), with
+// the row held in registers (VPT 8-wide vectors per thread): the row is read from memory once.
+// Narrow rows (the Wan-1.3B shape's 1536 columns) take 64-thread groups, so a CTA keeps four
+// rows in flight.  Mean and variance come from one group reduction of two sums in the
+// shifted-data form: sums of x - K and (x - K)^2 with K the row's first element, which keeps
+// E[(x-K)^2] - E[x-K]^2 free of cancellation however large the row's mean.
 template <bool F32IN>
 __device__ __forceinline__ void load_vec8(const void* xv, long long off, float (&v)[8]) {
   if (F32IN) {
@@ -126,25 +166,31 @@ __device__ __forceinline__ void load_vec8(const void* xv, long long off, float (
   }
 }
 
-template <bool F32IN, int VPT, int NT>
-__global__ void __launch_bounds__(NT, 1024 / NT) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
-                                                                   int cols, const float* __restrict__ mul,
-                                                                   float mul_bias, const float* __restrict__ add,
-                                                                   float eps) {
+constexpr int kNormThreads = 256;
+
+template <bool F32IN, int VPT, int TPR>
+__global__ void __launch_bounds__(kNormThreads, 4) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
+                                                                     int rows, int cols, const float* __restrict__ mul,
+                                                                     float mul_bias, const float* __restrict__ add,
+                                                                     float eps) {
   __shared__ float red[2][32];
-  const long long r0 = static_cast<long long>(blockIdx.x) * cols;
+  constexpr int kRows = kNormThreads / TPR;
+  const int t = threadIdx.x % TPR;
+  const long long row = static_cast<long long>(blockIdx.x) * kRows + threadIdx.x / TPR;
+  const bool live = row < rows;  // every thread still joins the group reduction's barriers
+  const long long r0 = (live ? row : 0) * cols;
   const int nvec = cols >> 3;
   const float K = F32IN ? static_cast<const float*>(xv)[r0] : bf16_to_f32(static_cast<const bf16*>(xv)[r0]);
   float v[VPT][8];
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
-    const int c = threadIdx.x + k * NT;
+    const int c = t + k * TPR;
     if (c < nvec) load_vec8<F32IN>(xv, r0 + 8LL * c, v[k]);
   }
   float s = 0.f, q = 0.f;
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
-    const int c = threadIdx.x + k * NT;
+    const int c = t + k * TPR;
     if (c < nvec) {
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
@@ -154,13 +200,14 @@ __global__ void __launch_bounds__(NT, 1024 / NT) row_norm_kernel(bf16* __restric
       }
     }
   }
-  const float2 t = block_sum2(s, q, red);
-  const float ms = t.x / cols;
+  const float2 sums = group_sum2<TPR>(s, q, red);
+  const float ms = sums.x / cols;
   const float mean = K + ms;
-  const float rstd = rsqrtf(fmaxf(t.y / cols - ms * ms, 0.f) + eps);
+  const float rstd = rsqrtf(fmaxf(sums.y / cols - ms * ms, 0.f) + eps);
+  if (!live) return;
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
-    const int c = threadIdx.x + k * NT;
+    const int c = t + k * TPR;
     if (c < nvec) {
       const float4* m4 = reinterpret_cast<const float4*>(mul) + 2 * c;
       const float4* a4 = reinterpret_cast<const float4*>(add) + 2 * c;
@@ -179,16 +226,23 @@ template <bool F32IN>
 cudaError_t row_norm_vpt(bf16* y, const void* x, int rows, int cols, const float* mul, float mul_bias,
                          const float* add, float eps, cudaStream_t s) {
   const int nvec = cols / 8;
-#define DFS_ROW_NORM(V, N) row_norm_kernel<F32IN, V, N><<<rows, N, 0, s>>>(y, x, cols, mul, mul_bias, add, eps)
-  if (nvec <= 5 * 128) {
+#define DFS_ROW_NORM(V, T)                                                                                    \
+  row_norm_kernel<F32IN, V, T><<<(rows + kNormThreads / (T) - 1) / (kNormThreads / (T)), kNormThreads, 0, s>>>( \
+      y, x, rows, cols, mul, mul_bias, add, eps)
+  if (nvec <= 4 * 64) {  // up to 2048 columns: 64 threads per row, four rows per CTA
+    switch ((nvec + 63) / 64) {
+      case 1: DFS_ROW_NORM(1, 64); break;
+      case 2: DFS_ROW_NORM(2, 64); break;
+      case 3: DFS_ROW_NORM(3, 64); break;
+      default: DFS_ROW_NORM(4, 64); break;
+    }
+  } else if (nvec <= 5 * 128) {  // up to 5120 columns: 128 threads per row
     switch ((nvec + 127) / 128) {
-      case 1: DFS_ROW_NORM(1, 128); break;
-      case 2: DFS_ROW_NORM(2, 128); break;
       case 3: DFS_ROW_NORM(3, 128); break;
       case 4: DFS_ROW_NORM(4, 128); break;
       default: DFS_ROW_NORM(5, 128); break;
     }
-  } else if (nvec <= 4 * 256) {
+  } else if (nvec <= 4 * 256) {  // up to 8192 columns: one row per CTA
     switch ((nvec + 255) / 256) {
       case 3: DFS_ROW_NORM(3, 256); break;
       default: DFS_ROW_NORM(4, 256); break;
@@ -217,17 +271,21 @@ struct QkParams {
   RopeTables t;
 };
 
-// One CTA per token row.  The row stays in registers as raw bf16 vectors (VPT 16-byte
-// vectors per thread), so several rows per SM are in flight at once.  The rotation of the
-// row's token (cos, sin per pair of a head, the same for every head) is built once in shared
-// memory from the per-band tables while the row loads, and the q and k statistics share one
-// reduction.
-template <int VPT>
-__global__ void __launch_bounds__(kQkThreads, 6) qk_norm_rope_kernel(const QkParams p) {
+// A group of TPR threads per token row, 256 / TPR rows per CTA (narrow rows, e.g. the
+// Wan-1.3B shape's 3072 q + k channels, take 64-thread groups and four rows per CTA).  The row
+// stays in registers as raw bf16 vectors (VPT 16-byte vectors per thread), so several rows per
+// SM are in flight at once.  The rotation of the row's token (cos, sin per pair of a head, the
+// same for every head) is built once per row in shared memory from the per-band tables while
+// the row loads, and the q and k statistics share one reduction.
+template <int VPT, int TPR>
+__global__ void __launch_bounds__(kQkThreads, 6) qk_norm_rope_kernel(const QkParams p, int rows) {
+  constexpr int kRows = kQkThreads / TPR;
   __shared__ float red[2][32];
-  __shared__ float rcos[64], rsin[64];
-  const long long row = blockIdx.x;
-  bf16* base = p.buf + row * p.ld;
+  __shared__ float rcos[kRows][64], rsin[kRows][64];
+  const int g = threadIdx.x / TPR, t = threadIdx.x % TPR;
+  const long long row = static_cast<long long>(blockIdx.x) * kRows + g;
+  const bool live = row < rows;  // every thread still joins the reductions' barriers
+  bf16* base = p.buf + (live ? row : 0) * p.ld;
   const int nvq = p.nq >> 3, nv = (p.nq + p.nk) >> 3;
   const int vph = p.head_dim >> 3;  // vectors per head (8 or 16); divides 32
   uint4 raw[VPT];
@@ -235,15 +293,16 @@ __global__ void __launch_bounds__(kQkThreads, 6) qk_norm_rope_kernel(const QkPar
   float sq = 0.f, sk = 0.f;
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
-    const int c = threadIdx.x + k * kQkThreads;
+    const int c = t + k * TPR;
     if (c < nv) raw[k] = reinterpret_cast<const uint4*>(base)[c];
   }
-  if (p.rope && threadIdx.x < (p.head_dim >> 1)) {
+  if (p.rope && t < (p.head_dim >> 1)) {
+    const long long tok = live ? row : 0;
     const int hw = p.t.grid_h * p.t.grid_w;
-    const int f = static_cast<int>(row / hw);
-    const int rem = static_cast<int>(row - static_cast<long long>(f) * hw);
+    const int f = static_cast<int>(tok / hw);
+    const int rem = static_cast<int>(tok - static_cast<long long>(f) * hw);
     const int yy = rem / p.t.grid_w, xx = rem - yy * p.t.grid_w;
-    const int j = threadIdx.x;
+    const int j = t;
     float cs, sn;
     if (j < p.t.p_t) {
       cs = __ldg(p.t.cos_t + f * p.t.p_t + j);
@@ -257,12 +316,12 @@ __global__ void __launch_bounds__(kQkThreads, 6) qk_norm_rope_kernel(const QkPar
       cs = __ldg(p.t.cos_w + xx * p.t.p_w + jj);
       sn = __ldg(p.t.sin_w + xx * p.t.p_w + jj);
     }
-    rcos[j] = cs;
-    rsin[j] = sn;
+    rcos[g][j] = cs;
+    rsin[g][j] = sn;
   }
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
-    const int c = threadIdx.x + k * kQkThreads;
+    const int c = t + k * TPR;
     float ss = 0.f;
     if (c < nv) {
       float v[8];
@@ -275,36 +334,37 @@ __global__ void __launch_bounds__(kQkThreads, 6) qk_norm_rope_kernel(const QkPar
   }
   float rq = 0.f, rk = 0.f;
   if (p.mode == 0) {
-    const float2 t = block_sum2(sq, sk, red);  // its barriers also publish the rotation table
-    rq = p.nq > 0 ? rsqrtf(t.x / p.nq + p.eps) : 0.f;
-    rk = p.nk > 0 ? rsqrtf(t.y / p.nk + p.eps) : 0.f;
+    const float2 sums = group_sum2<TPR>(sq, sk, red);  // its barriers also publish the rotation table
+    rq = p.nq > 0 ? rsqrtf(sums.x / p.nq + p.eps) : 0.f;
+    rk = p.nk > 0 ? rsqrtf(sums.y / p.nk + p.eps) : 0.f;
   } else {
     // per head: the vph threads holding one head are consecutive lanes of one warp
 #pragma unroll
     for (int k = 0; k < VPT; ++k) {
-      float t = hs[k];
-      for (int o = vph >> 1; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-      hs[k] = rsqrtf(t / p.head_dim + p.eps);
+      float h = hs[k];
+      for (int o = vph >> 1; o > 0; o >>= 1) h += __shfl_xor_sync(0xffffffffu, h, o);
+      hs[k] = rsqrtf(h / p.head_dim + p.eps);
     }
     if (p.rope) __syncthreads();
   }
+  if (!live) return;
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
-    const int c = threadIdx.x + k * kQkThreads;
+    const int c = t + k * TPR;
     if (c < nv) {
       const bool is_q = c < nvq;
       const int ch0 = (is_q ? c : c - nvq) * 8;  // channel within the q or k part
       const float r = p.mode == 0 ? (is_q ? rq : rk) : hs[k];
-      float v[8], g[8], o[8];
+      float v[8], gm[8], o[8];
       unpack_bf16x8(raw[k], v);
-      unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(is_q ? p.gq : p.gk) + (ch0 >> 3)), g);
+      unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(is_q ? p.gq : p.gk) + (ch0 >> 3)), gm);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) o[i] = v[i] * r * g[i];
+      for (int i = 0; i < 8; ++i) o[i] = v[i] * r * gm[i];
       if (p.rope) {
         const int j0 = (ch0 % p.head_dim) >> 1;  // first rotation pair of this vector
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          const float cs = rcos[j0 + i], sn = rsin[j0 + i];
+          const float cs = rcos[g][j0 + i], sn = rsin[g][j0 + i];
           const float a = o[2 * i], b = o[2 * i + 1];
           o[2 * i] = a * cs - b * sn;
           o[2 * i + 1] = a * sn + b * cs;
@@ -411,16 +471,37 @@ cudaError_t launch_qk_norm_rope(bf16* buf, long long ld, int rows, int nq, int n
   p.rope = rope != nullptr;
   if (rope) p.t = *rope; else memset(&p.t, 0, sizeof(p.t));
   if (head_dim > 128) return cudaErrorInvalidValue;  // the rotation table holds 64 pairs
-  const int vpt = ((nq + nk) / 8 + kQkThreads - 1) / kQkThreads;
-  switch (vpt) {
-    case 1: qk_norm_rope_kernel<1><<<rows, kQkThreads, 0, s>>>(p); break;
-    case 2: qk_norm_rope_kernel<2><<<rows, kQkThreads, 0, s>>>(p); break;
-    case 3: qk_norm_rope_kernel<3><<<rows, kQkThreads, 0, s>>>(p); break;
-    case 4: qk_norm_rope_kernel<4><<<rows, kQkThreads, 0, s>>>(p); break;
-    case 5: qk_norm_rope_kernel<5><<<rows, kQkThreads, 0, s>>>(p); break;
-    case 6: qk_norm_rope_kernel<6><<<rows, kQkThreads, 0, s>>>(p); break;
-    default: qk_norm_rope_kernel<8><<<rows, kQkThreads, 0, s>>>(p); break;
+  // thread group per row: 64 threads up to 256 vectors (2048 q + k channels), 128 up to 512,
+  // else 256; VPT vectors per thread (at most 4 in the narrow groups: 6 CTAs per SM leave a
+  // thread about 40 registers)
+  const int nv = (nq + nk) / 8;
+  const int tpr = nv <= 4 * 64 ? 64 : nv <= 4 * 128 ? 128 : 256;
+  const int vpt = (nv + tpr - 1) / tpr;
+  const int grid = (rows + kQkThreads / tpr - 1) / (kQkThreads / tpr);
+#define DFS_QK(V, T) qk_norm_rope_kernel<V, T><<<grid, kQkThreads, 0, s>>>(p, rows)
+  if (tpr == 64 || tpr == 128) {
+    switch (vpt + (tpr == 128 ? 4 : 0)) {
+      case 1: DFS_QK(1, 64); break;
+      case 2: DFS_QK(2, 64); break;
+      case 3: DFS_QK(3, 64); break;
+      case 4: DFS_QK(4, 64); break;
+      case 5: DFS_QK(1, 128); break;
+      case 6: DFS_QK(2, 128); break;
+      case 7: DFS_QK(3, 128); break;
+      default: DFS_QK(4, 128); break;
+    }
+  } else {
+    switch (vpt) {
+      case 1: DFS_QK(1, 256); break;
+      case 2: DFS_QK(2, 256); break;
+      case 3: DFS_QK(3, 256); break;
+      case 4: DFS_QK(4, 256); break;
+      case 5: DFS_QK(5, 256); break;
+      case 6: DFS_QK(6, 256); break;
+      default: DFS_QK(8, 256); break;
+    }
   }
+#undef DFS_QK
   return cudaGetLastError();
 }
 
