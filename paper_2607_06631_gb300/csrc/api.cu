@@ -74,6 +74,20 @@ bool make_map(CUtensorMap* m, const void* base, long long inner, long long outer
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tensor map of an fp32 [outer, inner] row-major matrix (leading dimension ld elements) with a
+// {32, 32} box and the 128-byte swizzle: the GEMM epilogue's TMA output stores.
+bool make_map_out_f32(CUtensorMap* m, const void* base, long long inner, long long outer, long long ld) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || inner <= 0 || outer <= 0) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 4};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 long long round_up(long long v, long long m) { return (v + m - 1) / m * m; }
 
 }  // namespace
@@ -560,6 +574,8 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     if (!make_map(&ma, P->attn, hd, N, hd, 64, 128) || !okbo) return fail(DFS_ECUDA, "tensor map (O) failed");
     S.g_o = gemm_args(P, ma, mb, N, d, hd, dfs::kEpiGatedRes, C.bo);
     S.g_o.out = P->x1; S.g_o.ldo = d; S.g_o.out_f32 = 1; S.g_o.ldr = d; S.g_o.res_f32 = 0;
+    if (!make_map_out_f32(&S.g_o.tma_out, P->x1, d, N, d)) return fail(DFS_ECUDA, "tensor map (O output) failed");
+    S.g_o.out_tma = 1;
     if (uni && (e = gather_kcols(S.g_o, S.pos_heads))) return e;
     dfs::AttnArgs& A = S.a_self;
     memset(&A, 0, sizeof(A));
@@ -608,6 +624,8 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     S.g_co = gemm_args(P, ma, mb, N, d, hcd, dfs::kEpiGatedRes, C.cbo);
     S.g_co.out = P->x1; S.g_co.ldo = d; S.g_co.out_f32 = 1; S.g_co.res = P->x1; S.g_co.ldr = d;
     S.g_co.res_f32 = 1; S.g_co.gate = nullptr;
+    if (!make_map_out_f32(&S.g_co.tma_out, P->x1, d, N, d)) return fail(DFS_ECUDA, "tensor map (cross O output) failed");
+    S.g_co.out_tma = 1;
     if (uni && (e = gather_kcols(S.g_co, S.pos_xheads))) return e;
     dfs::AttnArgs& A = S.a_cross;
     memset(&A, 0, sizeof(A));
@@ -1454,7 +1472,7 @@ dfs_status noalloc_forward(dfs_plan* P, int s, int l, const bf16* x, const bf16*
     DFS_CK(dfs::launch_attention(a, dh, st));
     dfs::GemmArgs o = S.g_o;
     if (!make_map(&o.tma_a, attn, hd, N, hd, 64, 128)) return fail(DFS_ECUDA, "tensor map (O) failed");
-    o.out = x1; o.res = x; o.gate = mod + 2 * d;
+    o.out = x1; o.res = x; o.gate = mod + 2 * d; o.out_tma = 0;
     DFS_CK(dfs::launch_gemm(o, P->num_sms, st));
   } else {
     DFS_CK(dfs::launch_bias_residual(x1, 1, x, 0, mod + 2 * d, C.bo, N, d, st));
@@ -1474,7 +1492,7 @@ dfs_status noalloc_forward(dfs_plan* P, int s, int l, const bf16* x, const bf16*
       DFS_CK(dfs::launch_attention(a, dh, st));
       dfs::GemmArgs o = S.g_co;
       if (!make_map(&o.tma_a, attn, hcd, N, hcd, 64, 128)) return fail(DFS_ECUDA, "tensor map (cross o) failed");
-      o.out = x1; o.res = x1;
+      o.out = x1; o.res = x1; o.out_tma = 0;
       DFS_CK(dfs::launch_gemm(o, P->num_sms, st));
     } else {
       DFS_CK(dfs::launch_bias_residual(x1, 1, x1, 1, nullptr, C.cbo, N, d, st));

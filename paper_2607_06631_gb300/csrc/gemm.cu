@@ -20,7 +20,10 @@
 //               where bases and row pitches allow, the accesses are 256-bit (one full 32-byte
 //               sector per row per instruction) to halve the number of L1 / L2 transactions.
 //               Short reductions use all 8 warps (two per TMEM lane quarter, 128 columns each),
-//               long ones warps 4..7 only (GemmArgs::epi_warps).
+//               long ones warps 4..7 only (GemmArgs::epi_warps).  The fp32 gated-residual output
+//               (x1) of full tiles goes out by TMA: each warp stages its 32 x 32 chunk in shared
+//               memory (128-byte swizzle) and one lane issues the tensor store, so the global
+//               writes leave as whole lines instead of 32 row pieces per instruction.
 // setmaxnreg splits the registers: 72 per thread in warpgroup 0, 216 in the epilogue
 // warpgroups (launch 384 x 168 = 128 x 72 + 256 x 216).
 // Ragged K (f_s is a multiple of 8, not of 64) is covered by TMA zero fill.
@@ -211,7 +214,10 @@ __device__ __forceinline__ void load_res_chunk(int res_f32, const char* rrow, in
 // output itself (in-place update): every element is still read by its own thread before
 // that thread writes it.
 template <int NCH>
-__device__ __forceinline__ void epilogue_gated_row(const GemmArgs& p, int row, int colb, uint32_t taddr) {
+__device__ __forceinline__ void epilogue_gated_row(const GemmArgs& p, int row, int colb, uint32_t taddr,
+                                                   uint8_t* stage) {
+  const int lane = threadIdx.x & 31;
+  const bool tma_out = p.out_tma && p.out_f32;
   const char* rrow = static_cast<const char*>(p.res) +
                      (static_cast<long long>(row) * p.ldr + colb) * (p.res_f32 ? 4 : 2);
   uint4 w[3][8];
@@ -264,7 +270,28 @@ __device__ __forceinline__ void epilogue_gated_row(const GemmArgs& p, int row, i
     }
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = fmaf(g[j], v[j], r[j]);
-    if (p.out_f32) {
+    if (tma_out) {
+      // this warp's 32 rows x 32 columns through its staging buffer (128 B swizzle: 16-byte
+      // piece q of row r at r * 128 + ((q ^ (r & 7)) << 4), conflict-free), stored by one TMA
+      // copy; the buffer is reused once the previous copy has read it
+      if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+      __syncwarp();
+      const uint32_t sb = smem_u32(stage) + lane * 128;
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(sb + ((q ^ (lane & 7)) << 4)), "f"(v[4 * q]),
+                     "f"(v[4 * q + 1]), "f"(v[4 * q + 2]), "f"(v[4 * q + 3])
+                     : "memory");
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) {
+        asm volatile(
+            "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];\n\t"
+            "cp.async.bulk.commit_group;" ::"l"(reinterpret_cast<uint64_t>(&p.tma_out)),
+            "r"(col0), "r"(row - lane), "r"(smem_u32(stage))
+            : "memory");
+      }
+    } else if (p.out_f32) {
       float* op = static_cast<float*>(p.out) + static_cast<long long>(row) * p.ldo + col0;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
@@ -295,7 +322,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + kGemmStages * kGemmABytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kGemmStages * kGemmStageBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kGemmStages * kGemmStageBytes + 8 * kGemmStageOut);
   uint64_t* empty = full + kGemmStages;
   uint64_t* tfull = empty + kGemmStages;
   uint64_t* tempty = tfull + 2;
@@ -415,6 +442,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     // with 8 epilogue warps each lane quarter's two warps take 128 columns of every tile; with
     // 4, warps 4..7 take all 256 and warps 8..11 have no work
     const int half = (warp - 4) >> 2;
+    uint8_t* stage = sB + kGemmStages * kGemmBBytes + (warp - 4) * kGemmStageOut;  // 1024-byte aligned
     const int c_lo = p.epi_warps == 8 ? 128 * half : 0, c_n = p.epi_warps == 8 ? 128 : kGemmBN;
     const bool idle = p.epi_warps != 8 && half == 1;
     const int r_in_tile = static_cast<int>(rank) * kGemmBM + sub * 32 + lane;
@@ -441,7 +469,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       // warp-uniform choice: the TMEM loads on both paths are warp-collective
       if (p.mode == kEpiGatedRes && kb > 0 && nt * kGemmBN + c_lo + c_n <= p.N && wide_ok &&
           __all_sync(0xffffffffu, row < p.M)) {
-        for (int c = c_lo; c < c_lo + c_n; c += 128) epilogue_gated_row<4>(p, row, nt * kGemmBN + c, tacc + c);
+        for (int c = c_lo; c < c_lo + c_n; c += 128) epilogue_gated_row<4>(p, row, nt * kGemmBN + c, tacc + c, stage);
       } else {
         for (int c = c_lo; c < c_lo + c_n; c += 32) {
           const int col0 = nt * kGemmBN + c;
@@ -471,6 +499,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
     }
+    // the output copies read this warp's staging buffer: complete before the CTA exits
+    if (lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    __syncwarp();
   }
 
   if (failed) drain_after_error();

@@ -27,7 +27,9 @@ static_assert((kGemmRegsControl + 2 * kGemmRegsEpilogue) * 32 <= 16384, "GEMM re
 constexpr int kGemmABytes = kGemmBM * kGemmBK * 2;
 constexpr int kGemmBBytes = kGemmBRows * kGemmBK * 2;
 constexpr int kGemmStageBytes = kGemmABytes + kGemmBBytes;
-constexpr int kGemmSmem = kGemmStages * kGemmStageBytes + 1024 + 256;
+constexpr int kGemmStageOut = 32 * 32 * 4;  // one epilogue warp's 32 x 32 fp32 output chunk (TMA store)
+constexpr int kGemmSmem = kGemmStages * kGemmStageBytes + 8 * kGemmStageOut + 1024 + 256;
+static_assert(kGemmSmem <= 227 * 1024, "GEMM shared memory exceeds a CTA's maximum");
 
 // How the B operand reaches shared memory.  kGatherNone reads B [N, K] as stored; the other
 // modes read a union weight matrix (the parameters retained at any step, Sec. 4.3) through
@@ -48,6 +50,7 @@ constexpr int kGemmMapMax = 512;  // entries: 3 * 8192 / 64 row groups, 8192 / 6
 struct GemmArgs {
   CUtensorMap tma_a;  // A [M, K], box {64, 128}, 128 B swizzle
   CUtensorMap tma_b;  // B [N, K], box {64, 128}, 128 B swizzle (see GatherMode for the others)
+  CUtensorMap tma_out;  // out_tma: fp32 output [M, ldo], box {32, 32}, 128 B swizzle
   int M, N, K;
   int mode;
   const bf16* bias;  // [N] or null
@@ -61,6 +64,7 @@ struct GemmArgs {
   long long ldr;
   int res_f32;
   const float* gate;  // [N] or null (gate = 1)
+  int out_tma;        // kEpiGatedRes, fp32 output: full tiles stored by TMA from shared memory
   int epi_warps;      // epilogue warps per CTA: 8 (two per TMEM lane quarter, 128 columns each) or 4
   int group;          // M tiles per raster group (tiles of one group sweep N together; odd groups
                       // sweep N backwards, so a group starts on the B bands the previous one ended on)
