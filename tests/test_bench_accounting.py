@@ -70,7 +70,7 @@ def test_reference_arm_prints_one_contract_line_on_the_tiny_block():
     assert d["impl"] == "reference" and d["unit"] == "TFLOP/s" and d["value"] > 0 and d["higher_is_better"]
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
-    assert "512 query rows" in d["cpu_baseline"]["sample"]
+    assert "whole MoM step" in d["cpu_baseline"]["sample"] and "512-token block" in d["cpu_baseline"]["sample"]
 
 
 def test_cpu_baseline_slice_extrapolation_on_a_small_block():
