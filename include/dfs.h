@@ -185,7 +185,7 @@ dfs_status dfs_block_forward_host_async(dfs_plan* plan, int step, int layer, con
  *     overlaps it.
  *   - Workspace of a (step, layer), with h = h_s head_dim, c = hc head_dim (cross heads,
  *     0 without cross-attention), f = f_s and every term rounded up to 256 bytes:
- *       24 dim + 2 N dim + 4 N h + 2 h ceil64(N) + 2 N max(h, c) + 4 N dim + 2 N f + 2 N c
+ *       24 dim + 2 N dim + 4 N h + 2 h ceil64(N) + 2 N max(h, c) + 4 N dim + 2 N ceil64(f) + 2 N c
  *     bytes; above 16 MiB (16777216 bytes) the call is rejected with DFS_EUNSUPPORTED and
  *     a message giving the need.
  * Errors: as dfs_block_forward_layer, plus DFS_EUNSUPPORTED. */
@@ -252,7 +252,7 @@ dfs_status dfs_plan_indices(const dfs_plan* plan, int step, int layer, int kind,
  * exported model (Sec. 3.2), i.e. the active parameters of step t gathered through I_t
  * (Sec. 4.3, Fig. 1(c)); bf16, row-major, leading dim *ld in elements.  which: 0 Wqkv [3 h_s dh, dim], 1 bqkv [3 h_s dh], 2 gq [h_s dh],
  * 3 gk [h_s dh], 4 Wo [dim, h_s dh], 5 W_up [f_s, dim], 6 b_up [f_s],
- * 7 W_down [dim, f_s]; cross: 8 cWq [hc dh, dim], 9 cbq, 10 cWkv [2 hc dh, dim],
+ * 7 W_down [dim, f_s] (leading dim f_s rounded up to a multiple of 64); cross: 8 cWq [hc dh, dim], 9 cbq, 10 cWkv [2 hc dh, dim],
  * 11 cbkv, 12 cgq, 13 cgk, 14 cWo [dim, hc dh].  A panel with zero rows or columns
  * returns *dev == NULL.  Under DFS_ENGINE_UNION the weight matrices (0, 4, 5, 7, 8, 10,
  * 14) have no per-step copy: they return their shape with *dev == NULL. */

@@ -469,14 +469,16 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
 
   // per-step panels; under the union engine only the vectors (the weight matrices are read
   // from the union through the maps) and, for the duration of plan creation, cWkv
+  // W_down [d, f_s] (7) gets a row pitch of whole 128-byte lines: f_s is a multiple of 8 only,
+  // and TMA rows that straddle L2 lines slowed its projection by a quarter
   auto mk = [&](int which, long long rows, long long cols) -> dfs_status {
     Panel& p = S.P[which];
-    p.rows = rows; p.cols = cols; p.ld = cols;
+    p.rows = rows; p.cols = cols; p.ld = which == 7 ? round_up(cols, 64) : cols;
     if (rows * cols == 0) return DFS_OK;
     const bool matrix = which == 0 || which == 4 || which == 5 || which == 7 || which == 8 || which == 10 ||
                         which == 14;
-    if (uni && matrix) return which == 10 ? alloc_temp(P, &p.p, rows * cols) : DFS_OK;
-    return alloc_weights(P, &p.p, rows * cols);
+    if (uni && matrix) return which == 10 ? alloc_temp(P, &p.p, rows * p.ld) : DFS_OK;
+    return alloc_weights(P, &p.p, rows * p.ld);
   };
   const bf16* wq = static_cast<const bf16*>(w.wq);
   const bf16* wk = static_cast<const bf16*>(w.wk);
@@ -509,8 +511,8 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     const int nch = static_cast<int>(S.chunks.size());
     if (!uni) {
       DFS_CK(dfs::launch_gather_rows(S.P[5].p, d, static_cast<const bf16*>(w.w_up), d, d_ffn_rows, fs, d, st));
-      DFS_CK(dfs::launch_gather_segs(S.P[7].p, fs, static_cast<const bf16*>(w.w_down), c.ffn_dim, d_chunks, nch,
-                                     d, st));
+      DFS_CK(dfs::launch_gather_segs(S.P[7].p, S.P[7].ld, static_cast<const bf16*>(w.w_down), c.ffn_dim, d_chunks,
+                                     nch, d, st));
     }
     DFS_CK(dfs::launch_gather_segs(S.P[6].p, 0, static_cast<const bf16*>(w.b_up), 0, d_chunks, nch, 1, st));
   }
@@ -591,11 +593,12 @@ dfs_status build_step_layer(dfs_plan* P, int s, int l, const dfs_layer_weights& 
     // union engine: the FFN panels live in the plan's per-forward scratch (same layout)
     const bf16* wup = uni ? P->ffn_up_s : S.P[5].p;
     const bf16* wdown = uni ? P->ffn_down_s : S.P[7].p;
+    const long long ldf = round_up(fs, 64);  // row pitch of h and W_down: whole 128-byte lines
     if (!make_map(&ma, P->xm, d, N, d, 64, 128) || !make_map(&mb, wup, d, fs, d, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (up) failed");
     S.g_up = gemm_args(P, ma, mb, N, fs, d, dfs::kEpiBiasGelu, S.P[6].p);
-    S.g_up.out = P->h; S.g_up.ldo = fs;
-    if (!make_map(&ma, P->h, fs, N, fs, 64, 128) || !make_map(&mb, wdown, fs, d, fs, 64, dfs::kGemmBRows))
+    S.g_up.out = P->h; S.g_up.ldo = ldf;
+    if (!make_map(&ma, P->h, fs, N, ldf, 64, 128) || !make_map(&mb, wdown, fs, d, ldf, 64, dfs::kGemmBRows))
       return fail(DFS_ECUDA, "tensor map (down) failed");
     S.g_down = gemm_args(P, ma, mb, N, d, fs, dfs::kEpiGatedRes, C.bdown);
     S.g_down.ldo = d; S.g_down.out_f32 = 0; S.g_down.res = P->x1; S.g_down.ldr = d; S.g_down.res_f32 = 1;
@@ -802,14 +805,14 @@ dfs_status create_impl(dfs_plan* P, const dfs_layer_weights* layers, const void*
   if ((e = alloc_n(P, &P->mod, 6LL * d)) || (e = alloc_n(P, &P->mod_base, 6LL * d * P->T)) ||
       (e = alloc_n(P, &P->xm, N * d)) || (e = alloc_n(P, &P->qk, N * 2 * hmax * dh)) ||
       (e = alloc_n(P, &P->vt, static_cast<long long>(hmax) * dh * P->vt_ld)) || (e = alloc_n(P, &P->attn, N * amax)) ||
-      (e = alloc_n(P, &P->x1, N * d)) || (e = alloc_n(P, &P->h, N * fmax)) ||
+      (e = alloc_n(P, &P->x1, N * d)) || (e = alloc_n(P, &P->h, N * round_up(fmax, 64))) ||
       (e = alloc_n(P, &P->qc, N * static_cast<long long>(hcmax) * dh)) || (e = alloc_n(P, &P->act[0], N * d)) ||
       (e = alloc_n(P, &P->act[1], N * d)) || (e = alloc_n(P, &P->stage_x, N * d)) ||
       (e = alloc_n(P, &P->stage_out, N * d)) || (e = alloc_n(P, &P->stage_t, d)))
     return e;
   if (hmax > 0) DFS_CK(cudaMemsetAsync(P->vt, 0, sizeof(bf16) * hmax * dh * P->vt_ld, st));
   if (P->uni && ((e = alloc_n(P, &P->ffn_up_s, static_cast<long long>(fmax) * d)) ||
-                 (e = alloc_n(P, &P->ffn_down_s, static_cast<long long>(fmax) * d))))
+                 (e = alloc_n(P, &P->ffn_down_s, round_up(fmax, 64) * d))))
     return e;
 
   // per layer: the union super-model; per (step, layer): index tables, compacted panels
@@ -845,12 +848,12 @@ dfs_status union_ffn_gather(dfs_plan* P, const StepLayer& S, int l, cudaStream_t
   const int d = P->cfg.dim, fs = S.f_s;
   if (profiled) {
     DFS_LAUNCH(DFS_K_GATHER, dfs::launch_gather_rows(P->ffn_up_s, d, U.wup.p, d, S.up_rows_u, fs, d, st));
-    DFS_LAUNCH(DFS_K_GATHER, dfs::launch_gather_segs(P->ffn_down_s, fs, U.wdown.p, U.wdown.ld, S.down_segs_u,
-                                                     fs / P->cfg.ffn_chunk, d, st));
+    DFS_LAUNCH(DFS_K_GATHER, dfs::launch_gather_segs(P->ffn_down_s, round_up(fs, 64), U.wdown.p, U.wdown.ld,
+                                                     S.down_segs_u, fs / P->cfg.ffn_chunk, d, st));
   } else {
     DFS_CK(dfs::launch_gather_rows(P->ffn_up_s, d, U.wup.p, d, S.up_rows_u, fs, d, st));
-    DFS_CK(dfs::launch_gather_segs(P->ffn_down_s, fs, U.wdown.p, U.wdown.ld, S.down_segs_u, fs / P->cfg.ffn_chunk,
-                                   d, st));
+    DFS_CK(dfs::launch_gather_segs(P->ffn_down_s, round_up(fs, 64), U.wdown.p, U.wdown.ld, S.down_segs_u,
+                                   fs / P->cfg.ffn_chunk, d, st));
   }
   return DFS_OK;
 }
@@ -1284,7 +1287,7 @@ dfs_status dfs_plan_workspace(const dfs_plan* P, int which, void** dev, int64_t*
     case 2: *dev = P->vt; *rows = hd; *cols = N; *ld = P->vt_ld; break;
     case 3: *dev = P->attn; *rows = N; *cols = hd; *ld = hd; break;
     case 4: *dev = P->x1; *rows = N; *cols = d; *ld = d; *dtype = 1; break;
-    case 5: *dev = P->h; *rows = N; *cols = S.f_s; *ld = S.f_s; break;
+    case 5: *dev = P->h; *rows = N; *cols = S.f_s; *ld = round_up(S.f_s, 64); break;
     case 6: *dev = P->mod; *rows = 6; *cols = d; *ld = d; *dtype = 1; break;
     default: return fail(DFS_EINVAL, "bad workspace id");
   }
@@ -1432,7 +1435,7 @@ dfs_status noalloc_forward(dfs_plan* P, int s, int l, const bf16* x, const bf16*
   };
   const long long o_mod = take(6LL * d * 4), o_xm = take(2LL * N * d), o_qk = take(2LL * N * 2 * hd),
                   o_vt = take(2LL * hd * vt_ld), o_attn = take(2LL * N * std::max(hd, hcd)),
-                  o_x1 = take(4LL * N * d), o_h = take(2LL * N * fs), o_qc = take(2LL * N * hcd);
+                  o_x1 = take(4LL * N * d), o_h = take(2LL * N * round_up(fs, 64)), o_qc = take(2LL * N * hcd);
   if (off > static_cast<long long>(kNoAllocScratchBytes))
     return fail(DFS_EUNSUPPORTED,
                 "this (step, layer) needs %lld bytes of scratch; the allocation-free forward has %zu",
@@ -1508,7 +1511,7 @@ dfs_status noalloc_forward(dfs_plan* P, int s, int l, const bf16* x, const bf16*
     u.out = h;
     DFS_CK(dfs::launch_gemm(u, P->num_sms, st));
     dfs::GemmArgs dn = S.g_down;
-    if (!make_map(&dn.tma_a, h, fs, N, fs, 64, 128)) return fail(DFS_ECUDA, "tensor map (down) failed");
+    if (!make_map(&dn.tma_a, h, fs, N, round_up(fs, 64), 64, 128)) return fail(DFS_ECUDA, "tensor map (down) failed");
     dn.out = out; dn.res = x1; dn.gate = mod + 5 * d;
     DFS_CK(dfs::launch_gemm(dn, P->num_sms, st));
   } else {

@@ -389,8 +389,15 @@ cudaError_t attention_prepare() {
   cudaError_t e = cudaFuncSetAttribute(attn_fwd_tcgen05<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        AttnLayout<64>::kSmem);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attn_fwd_tcgen05<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              AttnLayout<128>::kSmem);
+  e = cudaFuncSetAttribute(attn_fwd_tcgen05<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, AttnLayout<128>::kSmem);
+  if (e != cudaSuccess) return e;
+  // The softmax warpgroups' setmaxnreg.inc is satisfied only by the registers warpgroup 0
+  // releases, which assumes kRegsLaunch registers per thread at launch: a build that
+  // allocated fewer would make the increase wait forever, so it is refused here.
+  cudaFuncAttributes at64, at128;
+  if ((e = cudaFuncGetAttributes(&at64, attn_fwd_tcgen05<64>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&at128, attn_fwd_tcgen05<128>)) != cudaSuccess) return e;
+  return at64.numRegs == kRegsLaunch && at128.numRegs == kRegsLaunch ? cudaSuccess : cudaErrorNotSupported;
 }
 
 cudaError_t launch_attention(const AttnArgs& a, int head_dim, cudaStream_t s) {

@@ -516,7 +516,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
 }  // namespace
 
 cudaError_t gemm_prepare() {
-  return cudaFuncSetAttribute(gemm_bf16_tcgen05, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
+  cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tcgen05, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
+  if (e != cudaSuccess) return e;
+  // The epilogue warpgroups' setmaxnreg.inc is satisfied only by the registers warpgroup 0
+  // releases, which assumes kGemmRegsLaunch registers per thread at launch: a build that
+  // allocated fewer would make the increase wait forever, so it is refused here.
+  cudaFuncAttributes at;
+  if ((e = cudaFuncGetAttributes(&at, gemm_bf16_tcgen05)) != cudaSuccess) return e;
+  return at.numRegs == kGemmRegsLaunch ? cudaSuccess : cudaErrorNotSupported;
 }
 
 cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t s) {

@@ -157,7 +157,8 @@ def test_union_weight_memory_closed_form():
         idx = O.compact_indices(cfg, m, s, 0)
         hd, xd, fs = len(idx["heads"]) * dh, len(idx["xheads"]) * dh, len(idx["ffn_ch"])
         vec += 2 * (3 * hd + 2 * hd + fs + xd + 2 * xd + 2 * xd)         # bqkv gq gk b_up cbq cbkv cgq cgk
-        comp += 2 * (4 * hd * d + 2 * fs * d + 2 * xd * d + 2 * xd * d)   # wqkv wo w_up w_down cwq cwkv cwo
+        # wqkv wo w_up w_down cwq cwkv cwo; W_down's rows padded to a multiple of 64 elements
+        comp += 2 * (4 * hd * d + fs * d + d * ((fs + 63) // 64 * 64) + 2 * xd * d + 2 * xd * d)
     nu, nf, nx = len(u["heads"]) * dh, len(u["chunks"]) * C, len(u["xheads"]) * dh
     assert wc == comp + vec
     assert wu == 2 * (4 * nu * d + 2 * nf * d + 2 * nx * d) + vec

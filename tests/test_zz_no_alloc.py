@@ -106,5 +106,5 @@ def test_noalloc_forward_rejects_workspace_beyond_the_static_array():
     N, d, dh = cfg.n_tokens, cfg.dim, cfg.head_dim
     h, f = cfg.heads_kept[0][0] * dh, 8 * cfg.chunks_kept[0][0]
     need = (r(24 * d) + r(2 * N * d) + r(4 * N * h) + r(2 * h * ((N + 63) // 64 * 64)) + r(2 * N * h)
-            + r(4 * N * d) + r(2 * N * f))
+            + r(4 * N * d) + r(2 * N * ((f + 63) // 64 * 64)))
     assert ("needs %d bytes" % need) in str(e.value), (need, str(e.value))
