@@ -168,8 +168,38 @@ __device__ __forceinline__ void load_vec8(const void* xv, long long off, float (
 
 constexpr int kNormThreads = 256;
 
+// Raw words of one 8-element vector of the input row: fp32 keeps 8 floats, bf16 keeps the 4
+// packed words (half the registers, so more rows are in flight per SM).
+template <bool F32IN>
+struct RowVec {
+  uint32_t w[F32IN ? 8 : 4];
+};
+
+template <bool F32IN>
+__device__ __forceinline__ void load_raw8(const void* xv, long long off, RowVec<F32IN>& r) {
+  if constexpr (F32IN) {
+    const uint4* p = reinterpret_cast<const uint4*>(static_cast<const float*>(xv) + off);
+    const uint4 a = p[0], b = p[1];
+    r.w[0] = a.x; r.w[1] = a.y; r.w[2] = a.z; r.w[3] = a.w;
+    r.w[4] = b.x; r.w[5] = b.y; r.w[6] = b.z; r.w[7] = b.w;
+  } else {
+    const uint4 a = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(xv) + off);
+    r.w[0] = a.x; r.w[1] = a.y; r.w[2] = a.z; r.w[3] = a.w;
+  }
+}
+
+template <bool F32IN>
+__device__ __forceinline__ void unpack_raw8(const RowVec<F32IN>& r, float (&v)[8]) {
+  if constexpr (F32IN) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r.w[i]);
+  } else {
+    unpack_bf16x8(make_uint4(r.w[0], r.w[1], r.w[2], r.w[3]), v);
+  }
+}
+
 template <bool F32IN, int VPT, int TPR>
-__global__ void __launch_bounds__(kNormThreads, 4) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
+__global__ void __launch_bounds__(kNormThreads, F32IN ? 4 : 6) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
                                                                      int rows, int cols, const float* __restrict__ mul,
                                                                      float mul_bias, const float* __restrict__ add,
                                                                      float eps) {
@@ -181,20 +211,22 @@ __global__ void __launch_bounds__(kNormThreads, 4) row_norm_kernel(bf16* __restr
   const long long r0 = (live ? row : 0) * cols;
   const int nvec = cols >> 3;
   const float K = F32IN ? static_cast<const float*>(xv)[r0] : bf16_to_f32(static_cast<const bf16*>(xv)[r0]);
-  float v[VPT][8];
+  RowVec<F32IN> raw[VPT];
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
     const int c = t + k * TPR;
-    if (c < nvec) load_vec8<F32IN>(xv, r0 + 8LL * c, v[k]);
+    if (c < nvec) load_raw8<F32IN>(xv, r0 + 8LL * c, raw[k]);
   }
   float s = 0.f, q = 0.f;
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
     const int c = t + k * TPR;
     if (c < nvec) {
+      float v[8];
+      unpack_raw8<F32IN>(raw[k], v);
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const float d = v[k][i] - K;
+        const float d = v[i] - K;
         s += d;
         q = fmaf(d, d, q);
       }
@@ -214,9 +246,10 @@ __global__ void __launch_bounds__(kNormThreads, 4) row_norm_kernel(bf16* __restr
       const float4 m0 = __ldg(m4), m1 = __ldg(m4 + 1), a0 = __ldg(a4), a1 = __ldg(a4 + 1);
       const float mm[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
       const float aa[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-      float o[8];
+      float v[8], o[8];
+      unpack_raw8<F32IN>(raw[k], v);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) o[i] = fmaf((v[k][i] - mean) * rstd, mul_bias + mm[i], aa[i]);
+      for (int i = 0; i < 8; ++i) o[i] = fmaf((v[i] - mean) * rstd, mul_bias + mm[i], aa[i]);
       *reinterpret_cast<uint4*>(y + r0 + 8LL * c) = pack_bf16x8(o);
     }
   }
