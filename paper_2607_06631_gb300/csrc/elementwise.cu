@@ -310,8 +310,10 @@ struct QkParams {
 // SM are in flight at once.  The rotation of the row's token (cos, sin per pair of a head, the
 // same for every head) is built once per row in shared memory from the per-band tables while
 // the row loads, and the q and k statistics share one reduction.
+// Six CTAs per SM leave a thread about 40 registers, enough for up to five vectors; wider rows
+// (more than 10240 q + k channels) run four CTAs per SM so that their vectors stay in registers.
 template <int VPT, int TPR>
-__global__ void __launch_bounds__(kQkThreads, 6) qk_norm_rope_kernel(const QkParams p, int rows) {
+__global__ void __launch_bounds__(kQkThreads, VPT > 5 ? 4 : 6) qk_norm_rope_kernel(const QkParams p, int rows) {
   constexpr int kRows = kQkThreads / TPR;
   __shared__ float red[2][32];
   __shared__ float rcos[kRows][64], rsin[kRows][64];
