@@ -46,6 +46,7 @@ template <int TPR>
 __device__ __forceinline__ float2 group_sum2(float a, float b, float (*red)[32]) {
   a = warp_sum(a);
   b = warp_sum(b);
+  if constexpr (TPR == 32) return make_float2(a, b);  // one warp per group: no barrier
   constexpr int kWarps = TPR / 32;
   const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
   __syncthreads();
@@ -199,7 +200,7 @@ __device__ __forceinline__ void unpack_raw8(const RowVec<F32IN>& r, float (&v)[8
 }
 
 template <bool F32IN, int VPT, int TPR>
-__global__ void __launch_bounds__(kNormThreads, F32IN ? 4 : 6) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
+__global__ void __launch_bounds__(kNormThreads, (F32IN ? 4 : 6) - (VPT > 5 ? 1 : 0)) row_norm_kernel(bf16* __restrict__ y, const void* __restrict__ xv,
                                                                      int rows, int cols, const float* __restrict__ mul,
                                                                      float mul_bias, const float* __restrict__ add,
                                                                      float eps) {
@@ -262,7 +263,16 @@ cudaError_t row_norm_vpt(bf16* y, const void* x, int rows, int cols, const float
 #define DFS_ROW_NORM(V, T)                                                                                    \
   row_norm_kernel<F32IN, V, T><<<(rows + kNormThreads / (T) - 1) / (kNormThreads / (T)), kNormThreads, 0, s>>>( \
       y, x, rows, cols, mul, mul_bias, add, eps)
-  if (nvec <= 4 * 64) {  // up to 2048 columns: 64 threads per row, four rows per CTA
+  if (nvec <= 6 * 32) {  // up to 1536 columns: one warp per row, eight rows per CTA, no barrier
+    switch ((nvec + 31) / 32) {
+      case 1: DFS_ROW_NORM(1, 32); break;
+      case 2: DFS_ROW_NORM(2, 32); break;
+      case 3: DFS_ROW_NORM(3, 32); break;
+      case 4: DFS_ROW_NORM(4, 32); break;
+      case 5: DFS_ROW_NORM(5, 32); break;
+      default: DFS_ROW_NORM(6, 32); break;
+    }
+  } else if (nvec <= 4 * 64) {  // up to 2048 columns: 64 threads per row, four rows per CTA
     switch ((nvec + 63) / 64) {
       case 1: DFS_ROW_NORM(1, 64); break;
       case 2: DFS_ROW_NORM(2, 64); break;
