@@ -320,10 +320,16 @@ struct QkParams {
 // SM are in flight at once.  The rotation of the row's token (cos, sin per pair of a head, the
 // same for every head) is built once per row in shared memory from the per-band tables while
 // the row loads, and the q and k statistics share one reduction.
-// Six CTAs per SM leave a thread about 40 registers, enough for up to five vectors; wider rows
-// (more than 10240 q + k channels) run four CTAs per SM so that their vectors stay in registers.
+// CTAs per SM: six leave a thread about 40 registers, enough for up to five vectors of a
+// 256-thread row (four of a narrower group, whose rotation table costs a few more); more
+// vectors per thread take four or five CTAs per SM so that they stay in registers.
 template <int VPT, int TPR>
-__global__ void __launch_bounds__(kQkThreads, VPT > 5 ? 4 : 6) qk_norm_rope_kernel(const QkParams p, int rows) {
+constexpr int qk_min_blocks() {
+  return VPT > 5 ? 4 : (VPT == 5 && TPR != 256) ? 5 : 6;
+}
+
+template <int VPT, int TPR>
+__global__ void __launch_bounds__(kQkThreads, qk_min_blocks<VPT, TPR>()) qk_norm_rope_kernel(const QkParams p, int rows) {
   constexpr int kRows = kQkThreads / TPR;
   __shared__ float red[2][32];
   __shared__ float rcos[kRows][64], rsin[kRows][64];
@@ -516,23 +522,27 @@ cudaError_t launch_qk_norm_rope(bf16* buf, long long ld, int rows, int nq, int n
   p.rope = rope != nullptr;
   if (rope) p.t = *rope; else memset(&p.t, 0, sizeof(p.t));
   if (head_dim > 128) return cudaErrorInvalidValue;  // the rotation table holds 64 pairs
-  // thread group per row: 64 threads up to 256 vectors (2048 q + k channels), 128 up to 512,
-  // else 256; VPT vectors per thread (at most 4 in the narrow groups: 6 CTAs per SM leave a
-  // thread about 40 registers)
+  // thread group per row: 64 threads up to 384 vectors (3072 q + k channels), 128 up to 512,
+  // else 256; VPT vectors per thread
   const int nv = (nq + nk) / 8;
-  const int tpr = nv <= 4 * 64 ? 64 : nv <= 4 * 128 ? 128 : 256;
+  const int tpr = nv <= 6 * 64 ? 64 : nv <= 4 * 128 ? 128 : 256;
   const int vpt = (nv + tpr - 1) / tpr;
   const int grid = (rows + kQkThreads / tpr - 1) / (kQkThreads / tpr);
 #define DFS_QK(V, T) qk_norm_rope_kernel<V, T><<<grid, kQkThreads, 0, s>>>(p, rows)
-  if (tpr == 64 || tpr == 128) {
-    switch (vpt + (tpr == 128 ? 4 : 0)) {
+  if (tpr == 64) {
+    switch (vpt) {
       case 1: DFS_QK(1, 64); break;
       case 2: DFS_QK(2, 64); break;
       case 3: DFS_QK(3, 64); break;
       case 4: DFS_QK(4, 64); break;
-      case 5: DFS_QK(1, 128); break;
-      case 6: DFS_QK(2, 128); break;
-      case 7: DFS_QK(3, 128); break;
+      case 5: DFS_QK(5, 64); break;
+      default: DFS_QK(6, 64); break;
+    }
+  } else if (tpr == 128) {
+    switch (vpt) {
+      case 1: DFS_QK(1, 128); break;
+      case 2: DFS_QK(2, 128); break;
+      case 3: DFS_QK(3, 128); break;
       default: DFS_QK(4, 128); break;
     }
   } else {
